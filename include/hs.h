@@ -1,0 +1,229 @@
+/*
+ * hs.h -- checkpoint-aligned restore-and-resume for hybrid (full-attention +
+ * linear-attention) language models on one GB300 (sm_103a).
+ *
+ * The calls follow one resumed request:
+ *   1. hs_align_prefix                 strict-prefix lookup: pick the recurrent-state
+ *                                      checkpoint c the scheduler may credit (host).
+ *   2. hs_restore_kv_pages             scatter the cached KV pages of [0,c) from a device
+ *                                      staging pool into the paged KV cache by block table.
+ *   3. hs_restore_state                copy the float32 linear-attention state at c into the
+ *                                      live state.
+ *   4. hs_linattn_prefill_from_state   gated linear-attention prefill over the tail [c,N)
+ *                                      from that state, emitting state checkpoints.
+ *   5. hs_checkpoint_states            snapshot live states into checkpoint slots.
+ *
+ * Conventions shared by every call
+ *   - Every call returns hs_status.  HS_OK means the arguments passed host-side
+ *     validation and the work was enqueued; it does not wait for the GPU.
+ *   - The caller owns all memory.  The library never allocates or frees memory,
+ *     never synchronises a stream and keeps no mutable global state.
+ *   - "device" pointers point to GPU-visible memory of the current device; "host"
+ *     pointers are read by the host before the call returns.
+ *   - GPU work is enqueued on the caller's stream in argument order; calls on one
+ *     stream execute in issue order.
+ *   - Problems that only the GPU can see (a block id out of range, a misaligned
+ *     pointer read from a device pointer array, a bounded wait that ran out) are
+ *     reported through the optional device word d_err: the first kernel that
+ *     detects one stores an HS_DEVERR_* code there if it still holds 0.  Kernels
+ *     never clear it and never trap; the work item that failed is skipped.
+ *     Pass NULL to skip reporting.
+ *
+ * Data types: "bf16" arrays hold bfloat16 bit patterns (uint16_t); float is IEEE
+ * binary32.
+ */
+#ifndef HS_H
+#define HS_H
+
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum hs_status {
+    HS_OK = 0,
+    HS_ERR_INVALID_ARG = 1,   /* null pointer, negative or inconsistent size, unsorted list */
+    HS_ERR_MISALIGNED = 2,    /* pointer or byte size not a multiple of 16 bytes */
+    HS_ERR_UNSUPPORTED = 3,   /* shape outside what the kernels implement (see each call) */
+    HS_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed */
+    HS_ERR_DEVICE_CHECK = 5   /* reserved for callers that fold d_err into a status */
+} hs_status;
+
+/* codes a kernel may store into d_err */
+#define HS_DEVERR_NONE 0
+#define HS_DEVERR_BLOCK_OOB 1     /* block_table entry < 0 or >= num_blocks */
+#define HS_DEVERR_MISALIGNED 2    /* a pointer read from a device pointer array is not 16-byte aligned */
+#define HS_DEVERR_NULL 3          /* a pointer read from a device pointer array is NULL */
+#define HS_DEVERR_TIMEOUT 4       /* a bounded wait inside a kernel ran out */
+
+/* Largest batch accepted by hs_linattn_prefill_from_state. */
+#define HS_MAX_BATCH 512
+/* Chunk length of the prefill; checkpoint intervals are multiples of it. */
+#define HS_CHUNK 64
+
+/* Human-readable name of a status; never NULL. */
+const char *hs_status_string(hs_status s);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int32_t hs_version(void);
+
+/*
+ * hs_align_prefix -- strict-prefix checkpoint alignment (host only, no GPU).
+ *
+ * Paper: Section 2.2 (a state for prefix [0,B) continues from B, so the
+ * scheduler credits p = B; on a complete hit with every checkpoint cached,
+ * B = C*floor((N-1)/C)), Section 3.2 (the lookup query excludes the last known
+ * token, so a complete hit never credits N) and Table 4 / Figure 2.
+ *
+ * Chooses c = the largest b with b <= N-1, b <= hit_len, b % page_size == 0 and b
+ * either 0 (the empty prefix, always available) or listed in avail_ckpts.
+ *   N            prompt length in tokens, >= 1
+ *   hit_len      tokens of the prompt found in the external cache, 0 <= hit_len <= N
+ *   avail_ckpts  host, n_avail checkpoint positions (prefix lengths) held in the
+ *                cache, strictly increasing, each >= 0; entries above N are
+ *                ignored; may be NULL when n_avail == 0
+ *   page_size    KV page size in tokens, >= 1
+ *   c_out        host: the aligned checkpoint c (the scheduler credit p = c)
+ *   n_pages_out  host: c / page_size, the KV pages to restore per full layer
+ *   tail_out     host: N - c >= 1, tokens to recompute
+ * Errors: HS_ERR_INVALID_ARG (sizes, NULL outputs, unsorted or negative list).
+ */
+hs_status hs_align_prefix(int64_t N, int64_t hit_len, const int64_t *avail_ckpts, int32_t n_avail,
+                          int32_t page_size, int64_t *c_out, int64_t *n_pages_out,
+                          int64_t *tail_out);
+
+/*
+ * hs_restore_kv_pages -- scatter cached KV pages into the paged KV cache.
+ *
+ * Paper: Section 2.1 (attention cache entries travel with the checkpointed
+ * state), Section 5.2 (restored bytes per rank follow the chosen B) and
+ * Table 5 (H2D page transfers into poisoned destinations).
+ *
+ * For every layer l < n_layers and page j < n_pages:
+ *     cache_layers[l] + block_table[j]*page_bytes  <-  staging_layers[l] + j*page_bytes
+ * (page_bytes bytes).  Bytes of the cache outside the listed blocks are not
+ * written.
+ *   staging_layers  device array of n_layers device pointers, each to
+ *                   n_pages*page_bytes bytes laid out page after page
+ *   cache_layers    device array of n_layers device pointers, each to
+ *                   num_blocks*page_bytes bytes (one layer's paged cache)
+ *   block_table     device, n_pages int32 block ids; ids must be distinct (two equal
+ *                   ids race); an id outside [0,num_blocks) sets
+ *                   HS_DEVERR_BLOCK_OOB and that page is skipped
+ *   page_bytes      > 0, multiple of 16
+ * Every pointer in the arrays must be 16-byte aligned (else HS_DEVERR_MISALIGNED
+ * and the layer is skipped).  n_layers == 0 or n_pages == 0 is a no-op.
+ * Errors: HS_ERR_INVALID_ARG, HS_ERR_MISALIGNED (page_bytes), HS_ERR_CUDA.
+ */
+hs_status hs_restore_kv_pages(const void *const *staging_layers, void *const *cache_layers,
+                              int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                              int64_t page_bytes, int64_t num_blocks, int32_t *d_err,
+                              cudaStream_t stream);
+
+/*
+ * hs_restore_state -- restore recurrent states from checkpoint slots.
+ *
+ * Paper: Section 1 (a state updated in place cannot be rebuilt by reducing a
+ * token count; it must be restored for the credited prefix) and Section 2.2.
+ *
+ * dst_slots[i][0..floats_each) <- src_slots[i][0..floats_each) for i < n, bit-exact.
+ *   src_slots  device array of n device pointers (checkpoint slots; only read)
+ *   dst_slots  device array of n device pointers (live states)
+ * Slots may have any 4-byte alignment (16-byte aligned slots take the vector
+ * path); NULL entries set HS_DEVERR_NULL and are skipped; slots must not overlap.
+ * Errors: HS_ERR_INVALID_ARG, HS_ERR_CUDA.
+ */
+hs_status hs_restore_state(const float *const *src_slots, float *const *dst_slots, int32_t n,
+                           int64_t floats_each, int32_t *d_err, cudaStream_t stream);
+
+/*
+ * hs_checkpoint_states -- snapshot live recurrent states into checkpoint slots.
+ *
+ * Paper: Table 1 (state checkpoints every C tokens) and Section 6 (a stored
+ * checkpoint is an immutable payload).  Same contract as hs_restore_state with
+ * src = live states and dst = checkpoint slots; restore never writes slots.
+ */
+hs_status hs_checkpoint_states(const float *const *live_states, float *const *ckpt_slots,
+                               int32_t n, int64_t floats_each, int32_t *d_err,
+                               cudaStream_t stream);
+
+/* Which kernel hs_linattn_prefill_from_state runs. */
+typedef enum hs_linattn_kernel {
+    HS_LINATTN_AUTO = 0,       /* the library's choice for the shape */
+    HS_LINATTN_RECURRENT = 1,  /* per-token recurrence, CUDA cores */
+    HS_LINATTN_CHUNKED_TC = 2  /* chunked form on tcgen05 tensor cores */
+} hs_linattn_kernel;
+
+typedef struct hs_linattn_shape {
+    int32_t batch;         /* independent problems: requests, or (request, layer) pairs */
+    int32_t n_heads;       /* heads per problem */
+    int32_t d_k;           /* key/query width: 64 or 128 */
+    int32_t d_v;           /* value width: equal to d_k */
+    int64_t max_tokens;    /* token extent T of q/k/v/log_g/o per problem (>= every n_tokens) */
+    int32_t kernel;        /* hs_linattn_kernel */
+    int32_t reserved;      /* must be 0 */
+} hs_linattn_shape;
+
+/*
+ * hs_linattn_prefill_from_state -- gated linear-attention prefill from a
+ * restored state.
+ *
+ * Paper: Section 2.2 (continue from the state of [0,B) over the suffix
+ * [B,N)), Section 4.1 and Table 2 (matched checkpoint schedule), Section 4.2 /
+ * Table 3 (fixed kernel configuration).  The paper runs its linear layers on
+ * the FLA kernels without printing their recurrence; this call implements
+ *     S_t = diag(g_t) S_{t-1} + k_t v_t^T,   o_t = q_t S_t,   g_t = exp(a_t)
+ * with a_t <= 0 the per-dimension log-gates (a very negative a, e.g. -1e4,
+ * is a zero gate).
+ *
+ * For problem b, token t < n_tokens[b] of q/k/v/log_g/o is absolute position
+ * pos0[b] + t.  state[b] holds on entry the state of prefix [0,pos0[b]) and on
+ * return that of [0,pos0[b]+n_tokens[b]).  Work is split into chunks of
+ * HS_CHUNK tokens on the absolute position grid and every chunk is a fixed
+ * function of its inputs and its incoming state, so resuming at a multiple of
+ * HS_CHUNK reproduces a full recomputation bit for bit (same kernel choice).
+ *
+ *   shp        host; batch in [0, HS_MAX_BATCH]; d_k == d_v in {64,128}
+ *   q, k       device bf16 [batch][max_tokens][n_heads][d_k]
+ *   v          device bf16 [batch][max_tokens][n_heads][d_v]
+ *   log_g      device float [batch][max_tokens][n_heads][d_k]
+ *   o          device float [batch][max_tokens][n_heads][d_v]; rows t >= n_tokens[b]
+ *              are not written
+ *   state      device float [batch][n_heads][d_k][d_v], row index = key dimension
+ *   pos0       host int64 [batch], >= 0
+ *   n_tokens   host int32 [batch], 0 <= n_tokens[b] <= max_tokens
+ *   ckpt_interval  C: 0 (no checkpoints) or a positive multiple of HS_CHUNK
+ *   ckpt_slots device array of device pointers or NULL (no checkpoints written).
+ *              Problem b emits one checkpoint for every multiple m*C in
+ *              (pos0[b], pos0[b]+n_tokens[b]]: the state of prefix [0,m*C), float
+ *              [n_heads][d_k][d_v].  Slots are listed problem by problem, in
+ *              position order; hs_linattn_num_checkpoints gives the count.  Each
+ *              slot must be 16-byte aligned (else HS_DEVERR_MISALIGNED, not written).
+ *   d_err      optional device int32 (see conventions)
+ * All of q, k, v, log_g, o, state must be 16-byte aligned.  q/k/v/log_g are only
+ * read; o, state and the slots must not overlap the inputs or each other.
+ * Errors: HS_ERR_INVALID_ARG, HS_ERR_MISALIGNED, HS_ERR_UNSUPPORTED (d_k/d_v,
+ * ckpt_interval not a multiple of HS_CHUNK, batch > HS_MAX_BATCH), HS_ERR_CUDA.
+ */
+hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint16_t *q,
+                                        const uint16_t *k, const uint16_t *v, const float *log_g,
+                                        float *o, float *state, const int64_t *pos0,
+                                        const int32_t *n_tokens, int32_t ckpt_interval,
+                                        float *const *ckpt_slots, int32_t *d_err,
+                                        cudaStream_t stream);
+
+/*
+ * hs_linattn_num_checkpoints -- number of checkpoint slots the prefill above
+ * writes for these arguments (host only): the sum over b of
+ * floor((pos0[b]+n_tokens[b])/C) - floor(pos0[b]/C), 0 when C == 0.
+ */
+hs_status hs_linattn_num_checkpoints(int32_t batch, const int64_t *pos0, const int32_t *n_tokens,
+                                     int32_t ckpt_interval, int64_t *total_out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HS_H */

@@ -1,0 +1,233 @@
+// C-ABI entry points of libhs: host-side validation, then one launch per call.
+// Validation happens before any CUDA runtime call, so argument errors are
+// reported without touching the GPU.
+#include <cstring>
+
+#include "hs_internal.cuh"
+
+namespace {
+
+inline bool misaligned16(const void *p)
+{
+    return (reinterpret_cast<uintptr_t>(p) & 15u) != 0;
+}
+
+inline hs_status cuda_status(cudaError_t e)
+{
+    return e == cudaSuccess ? HS_OK : HS_ERR_CUDA;
+}
+
+hs_status sm_count(int *out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return HS_ERR_CUDA;
+    if (cudaDeviceGetAttribute(out, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return HS_ERR_CUDA;
+    return HS_OK;
+}
+
+hs_status copy_slots(const float *const *src, float *const *dst, int32_t n, int64_t floats_each,
+                     int32_t *d_err, cudaStream_t stream)
+{
+    if (n < 0 || floats_each < 0)
+        return HS_ERR_INVALID_ARG;
+    if (n == 0 || floats_each == 0)
+        return HS_OK;
+    if (src == nullptr || dst == nullptr)
+        return HS_ERR_INVALID_ARG;
+    int sms = 0;
+    hs_status st = sm_count(&sms);
+    if (st != HS_OK)
+        return st;
+    return cuda_status(hs::launch_slot_copy(src, dst, n, floats_each, d_err, sms, stream));
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *hs_status_string(hs_status s)
+{
+    switch (s) {
+    case HS_OK: return "HS_OK";
+    case HS_ERR_INVALID_ARG: return "HS_ERR_INVALID_ARG: invalid argument";
+    case HS_ERR_MISALIGNED: return "HS_ERR_MISALIGNED: pointer or size not 16-byte aligned";
+    case HS_ERR_UNSUPPORTED: return "HS_ERR_UNSUPPORTED: shape not implemented";
+    case HS_ERR_CUDA: return "HS_ERR_CUDA: CUDA runtime call or launch failed";
+    case HS_ERR_DEVICE_CHECK: return "HS_ERR_DEVICE_CHECK: a kernel reported an error";
+    }
+    return "unknown hs_status";
+}
+
+int32_t hs_version(void)
+{
+    return 100;  // 0.1.0
+}
+
+hs_status hs_align_prefix(int64_t N, int64_t hit_len, const int64_t *avail_ckpts, int32_t n_avail,
+                          int32_t page_size, int64_t *c_out, int64_t *n_pages_out,
+                          int64_t *tail_out)
+{
+    if (N < 1 || hit_len < 0 || hit_len > N || page_size < 1 || n_avail < 0)
+        return HS_ERR_INVALID_ARG;
+    if (c_out == nullptr || n_pages_out == nullptr || tail_out == nullptr)
+        return HS_ERR_INVALID_ARG;
+    if (n_avail > 0 && avail_ckpts == nullptr)
+        return HS_ERR_INVALID_ARG;
+    for (int32_t i = 0; i < n_avail; ++i) {
+        if (avail_ckpts[i] < 0 || (i > 0 && avail_ckpts[i] <= avail_ckpts[i - 1]))
+            return HS_ERR_INVALID_ARG;
+    }
+    // strict prefix: the query excludes the last prompt token and stops at the hit
+    const int64_t bound = (N - 1 < hit_len) ? N - 1 : hit_len;
+    // largest listed position <= bound (binary search), then walk down to a page boundary
+    int32_t lo = 0, hi = n_avail;  // first index with value > bound
+    while (lo < hi) {
+        const int32_t mid = lo + (hi - lo) / 2;
+        if (avail_ckpts[mid] <= bound)
+            lo = mid + 1;
+        else
+            hi = mid;
+    }
+    int64_t c = 0;
+    for (int32_t i = lo - 1; i >= 0; --i) {
+        if (avail_ckpts[i] % page_size == 0) {
+            c = avail_ckpts[i];
+            break;
+        }
+    }
+    *c_out = c;
+    *n_pages_out = c / page_size;
+    *tail_out = N - c;
+    return HS_OK;
+}
+
+hs_status hs_restore_kv_pages(const void *const *staging_layers, void *const *cache_layers,
+                              int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                              int64_t page_bytes, int64_t num_blocks, int32_t *d_err,
+                              cudaStream_t stream)
+{
+    if (n_layers < 0 || n_pages < 0 || page_bytes <= 0 || num_blocks < 0)
+        return HS_ERR_INVALID_ARG;
+    if (page_bytes % 16 != 0)
+        return HS_ERR_MISALIGNED;
+    if (n_layers == 0 || n_pages == 0)
+        return HS_OK;
+    if (staging_layers == nullptr || cache_layers == nullptr || block_table == nullptr)
+        return HS_ERR_INVALID_ARG;
+    if ((int64_t)n_pages > num_blocks)
+        return HS_ERR_INVALID_ARG;  // block ids must be distinct
+    int sms = 0;
+    hs_status st = sm_count(&sms);
+    if (st != HS_OK)
+        return st;
+    return cuda_status(hs::launch_kv_scatter(staging_layers, cache_layers, n_layers, block_table,
+                                             n_pages, page_bytes, num_blocks, d_err, sms, stream));
+}
+
+hs_status hs_restore_state(const float *const *src_slots, float *const *dst_slots, int32_t n,
+                           int64_t floats_each, int32_t *d_err, cudaStream_t stream)
+{
+    return copy_slots(src_slots, dst_slots, n, floats_each, d_err, stream);
+}
+
+hs_status hs_checkpoint_states(const float *const *live_states, float *const *ckpt_slots,
+                               int32_t n, int64_t floats_each, int32_t *d_err,
+                               cudaStream_t stream)
+{
+    return copy_slots(live_states, ckpt_slots, n, floats_each, d_err, stream);
+}
+
+hs_status hs_linattn_num_checkpoints(int32_t batch, const int64_t *pos0, const int32_t *n_tokens,
+                                     int32_t ckpt_interval, int64_t *total_out)
+{
+    if (batch < 0 || ckpt_interval < 0 || total_out == nullptr)
+        return HS_ERR_INVALID_ARG;
+    if (batch > 0 && (pos0 == nullptr || n_tokens == nullptr))
+        return HS_ERR_INVALID_ARG;
+    int64_t total = 0;
+    for (int32_t b = 0; b < batch; ++b) {
+        if (pos0[b] < 0 || n_tokens[b] < 0)
+            return HS_ERR_INVALID_ARG;
+        if (ckpt_interval > 0 && n_tokens[b] > 0)
+            total += (pos0[b] + n_tokens[b]) / ckpt_interval - pos0[b] / ckpt_interval;
+    }
+    *total_out = total;
+    return HS_OK;
+}
+
+hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint16_t *q,
+                                        const uint16_t *k, const uint16_t *v, const float *log_g,
+                                        float *o, float *state, const int64_t *pos0,
+                                        const int32_t *n_tokens, int32_t ckpt_interval,
+                                        float *const *ckpt_slots, int32_t *d_err,
+                                        cudaStream_t stream)
+{
+    if (shp == nullptr)
+        return HS_ERR_INVALID_ARG;
+    const hs_linattn_shape s = *shp;
+    if (s.batch < 0 || s.n_heads < 1 || s.max_tokens < 0 || s.reserved != 0)
+        return HS_ERR_INVALID_ARG;
+    if (s.kernel != HS_LINATTN_AUTO && s.kernel != HS_LINATTN_RECURRENT &&
+        s.kernel != HS_LINATTN_CHUNKED_TC)
+        return HS_ERR_INVALID_ARG;
+    if (s.d_k != s.d_v || (s.d_k != 64 && s.d_k != 128))
+        return HS_ERR_UNSUPPORTED;
+    if (s.batch > HS_MAX_BATCH)
+        return HS_ERR_UNSUPPORTED;
+    if (ckpt_interval < 0)
+        return HS_ERR_INVALID_ARG;
+    if (ckpt_interval % HS_CHUNK != 0)
+        return HS_ERR_UNSUPPORTED;
+    if (s.batch == 0)
+        return HS_OK;
+    if (pos0 == nullptr || n_tokens == nullptr || state == nullptr)
+        return HS_ERR_INVALID_ARG;
+    bool any_tokens = false;
+    for (int32_t b = 0; b < s.batch; ++b) {
+        if (pos0[b] < 0 || n_tokens[b] < 0 || (int64_t)n_tokens[b] > s.max_tokens)
+            return HS_ERR_INVALID_ARG;
+        if (pos0[b] > ((int64_t)1 << 40))
+            return HS_ERR_INVALID_ARG;
+        any_tokens = any_tokens || n_tokens[b] > 0;
+    }
+    if (!any_tokens)
+        return HS_OK;
+    if (q == nullptr || k == nullptr || v == nullptr || log_g == nullptr || o == nullptr)
+        return HS_ERR_INVALID_ARG;
+    if (misaligned16(q) || misaligned16(k) || misaligned16(v) || misaligned16(log_g) ||
+        misaligned16(o) || misaligned16(state))
+        return HS_ERR_MISALIGNED;
+
+    hs::GlaParams p;
+    std::memset(&p, 0, sizeof p);
+    p.q = q;
+    p.k = k;
+    p.v = v;
+    p.log_g = log_g;
+    p.o = o;
+    p.state = state;
+    p.ckpt_slots = (ckpt_interval > 0) ? ckpt_slots : nullptr;
+    p.d_err = d_err;
+    p.max_tokens = s.max_tokens;
+    p.batch = s.batch;
+    p.n_heads = s.n_heads;
+    p.ckpt_interval = (p.ckpt_slots != nullptr) ? ckpt_interval : 0;
+    int64_t base = 0;
+    for (int32_t b = 0; b < s.batch; ++b) {
+        p.pos0[b] = pos0[b];
+        p.n_tokens[b] = n_tokens[b];
+        p.ck_base[b] = (int32_t)base;
+        if (p.ckpt_interval > 0 && n_tokens[b] > 0)
+            base += (pos0[b] + n_tokens[b]) / p.ckpt_interval - pos0[b] / p.ckpt_interval;
+    }
+    if (base > INT32_MAX)
+        return HS_ERR_INVALID_ARG;
+
+    if (s.kernel == HS_LINATTN_CHUNKED_TC)
+        return cuda_status(hs::launch_gla_chunked_tc(p, s.d_k, stream));
+    return cuda_status(hs::launch_gla_recurrent(p, s.d_k, stream));
+}
+
+}  // extern "C"

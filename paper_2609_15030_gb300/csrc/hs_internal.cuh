@@ -1,0 +1,47 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "hs.h"
+
+namespace hs {
+
+// First detected device-side problem wins; kernels never clear the word.
+__device__ __forceinline__ void report(int32_t *d_err, int32_t code)
+{
+    if (d_err != nullptr)
+        atomicCAS(d_err, 0, code);
+}
+
+// Per-call description of a linear-attention prefill, passed by value to the kernels.
+struct GlaParams {
+    const uint16_t *q;
+    const uint16_t *k;
+    const uint16_t *v;
+    const float *log_g;
+    float *o;
+    float *state;
+    float *const *ckpt_slots;  // device array or nullptr
+    int32_t *d_err;
+    int64_t max_tokens;
+    int32_t batch;
+    int32_t n_heads;
+    int32_t ckpt_interval;     // 0: none
+    int32_t pad_;
+    int64_t pos0[HS_MAX_BATCH];
+    int32_t n_tokens[HS_MAX_BATCH];
+    int32_t ck_base[HS_MAX_BATCH];  // index of the problem's first slot in ckpt_slots
+};
+
+// launchers (return the launch's cudaError_t)
+cudaError_t launch_kv_scatter(const void *const *staging, void *const *cache, int32_t n_layers,
+                              const int32_t *bt, int32_t n_pages, int64_t page_bytes,
+                              int64_t num_blocks, int32_t *d_err, int sm_count, cudaStream_t s);
+cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t n,
+                             int64_t floats_each, int32_t *d_err, int sm_count, cudaStream_t s);
+cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);
+cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s);
+
+}  // namespace hs

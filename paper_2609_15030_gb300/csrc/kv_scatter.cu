@@ -1,0 +1,94 @@
+// Block-table scatter of KV pages from a device staging pool into the paged
+// KV cache (restoring the attention cache entries of the credited prefix,
+// Section 2.1 and Section 5.2 of the paper).
+//
+// Pure HBM copy: every page is a contiguous run of page_bytes bytes on both
+// sides, so each CTA moves whole pages with 16-byte vector loads and stores.
+// Loads bypass L1 and stores are streaming (evict-first): neither side is
+// reused by this kernel.  Several 16-byte loads are in flight per thread
+// before the first store so that the copy is limited by bandwidth, not by
+// load latency.  The grid is a whole number of waves over the SMs and
+// strides over (layer, page) units with pages of one layer adjacent, so
+// reads from the staging pool are sequential.
+#include "hs_internal.cuh"
+
+namespace hs {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 8;
+
+__device__ __forceinline__ uint4 ld_stream(const uint4 *p)
+{
+    return __ldcs(p);
+}
+
+__device__ __forceinline__ void st_stream(uint4 *p, const uint4 &v)
+{
+    __stcs(p, v);
+}
+
+__global__ void __launch_bounds__(kThreads)
+kv_scatter_kernel(const void *const *staging, void *const *cache, int32_t n_layers,
+                  const int32_t *bt, int32_t n_pages, int64_t page_vecs, int64_t num_blocks,
+                  int32_t *d_err)
+{
+    const int64_t units = (int64_t)n_layers * n_pages;
+    for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+        const int32_t l = (int32_t)(u / n_pages);
+        const int32_t j = (int32_t)(u - (int64_t)l * n_pages);
+        const uint4 *src = static_cast<const uint4 *>(staging[l]);
+        uint4 *dst = static_cast<uint4 *>(cache[l]);
+        const int32_t blk = bt[j];
+        if (src == nullptr || dst == nullptr) {
+            if (threadIdx.x == 0)
+                report(d_err, HS_DEVERR_NULL);
+            continue;
+        }
+        if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u) != 0) {
+            if (threadIdx.x == 0)
+                report(d_err, HS_DEVERR_MISALIGNED);
+            continue;
+        }
+        if (blk < 0 || (int64_t)blk >= num_blocks) {
+            if (threadIdx.x == 0)
+                report(d_err, HS_DEVERR_BLOCK_OOB);
+            continue;
+        }
+        src += (int64_t)j * page_vecs;
+        dst += (int64_t)blk * page_vecs;
+        for (int64_t base = threadIdx.x; base < page_vecs; base += (int64_t)kThreads * kUnroll) {
+            uint4 r[kUnroll];
+#pragma unroll
+            for (int x = 0; x < kUnroll; ++x) {
+                const int64_t i = base + (int64_t)x * kThreads;
+                if (i < page_vecs)
+                    r[x] = ld_stream(src + i);
+            }
+#pragma unroll
+            for (int x = 0; x < kUnroll; ++x) {
+                const int64_t i = base + (int64_t)x * kThreads;
+                if (i < page_vecs)
+                    st_stream(dst + i, r[x]);
+            }
+        }
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_kv_scatter(const void *const *staging, void *const *cache, int32_t n_layers,
+                              const int32_t *bt, int32_t n_pages, int64_t page_bytes,
+                              int64_t num_blocks, int32_t *d_err, int sm_count, cudaStream_t s)
+{
+    const int64_t units = (int64_t)n_layers * n_pages;
+    // 8 resident CTAs of 256 threads per SM; at most 4 waves, never more CTAs than units
+    int64_t grid = (int64_t)sm_count * 8 * 4;
+    if (grid > units)
+        grid = units;
+    kv_scatter_kernel<<<(unsigned)grid, kThreads, 0, s>>>(staging, cache, n_layers, bt, n_pages,
+                                                          page_bytes / 16, num_blocks, d_err);
+    return cudaGetLastError();
+}
+
+}  // namespace hs

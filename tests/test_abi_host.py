@@ -1,0 +1,175 @@
+"""Host-only checks of the C-ABI library (no GPU needed).
+
+* libhs.so loads and exports every function include/hs.h declares;
+* hs_align_prefix (host integer code) matches the oracle bit-exactly;
+* every argument error is reported before any CUDA call.
+"""
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+import paper_2609_15030_gb300 as hs
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2609_15030_gb300 import build
+    build.build()
+
+
+def _declared():
+    txt = open(os.path.join(ROOT, "include", "hs.h")).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(hs_[a-z0-9_]+)\s*\(", txt)))
+
+
+def test_exports_every_declared_symbol():
+    import ctypes
+    lib = ctypes.CDLL(hs.LIB_PATH)
+    names = _declared()
+    assert "hs_linattn_prefill_from_state" in names and len(names) >= 8
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(hs.EXPORTED) <= set(names)
+
+
+def test_status_strings_and_version():
+    for s in range(6):
+        assert hs.hs_status_string(s).startswith("HS_")
+    assert "unknown" in hs.hs_status_string(99)
+    assert hs.hs_version() >= 100
+
+
+def _rows():
+    out = []
+    for line in open(os.path.join(ROOT, "tests", "golden", "table4_alignment.txt")):
+        line = line.strip()
+        if line and not line.startswith("#"):
+            out.append([int(x) for x in line.split()])
+    return out
+
+
+def test_align_table4():
+    C = 1792
+    for N, _, _, B_after, suffix in _rows():
+        c, npg, tail = hs.hs_align_prefix(N, N, list(range(C, N + 1, C)), 16)
+        assert (c, tail) == (B_after, suffix)
+        assert npg == c // 16
+
+
+def test_align_matches_oracle_bit_exact():
+    rng = np.random.default_rng(77)
+    for _ in range(4000):
+        N = int(rng.integers(1, 400))
+        hit = int(rng.integers(0, N + 1))
+        P = int(rng.choice([1, 2, 16, 32]))
+        avail = sorted(set(int(x) for x in rng.integers(0, N + 50, size=int(rng.integers(0, 20)))))
+        assert hs.hs_align_prefix(N, hit, avail, P) == oracle.align_prefix(N, hit, avail, P)
+
+
+def test_align_config_lengths():
+    # sweep / hybrid / long-context lengths, complete and partial (L-37) hits
+    for C, P, Ls in ((512, 16, range(512, 4609, 512)), (256, 16, range(512, 4609, 512)),
+                     (512, 32, (16384, 32768, 65536))):
+        for L in Ls:
+            for hit in (L, L - 37):
+                av = list(range(C, L + 1, C))
+                assert hs.hs_align_prefix(L, hit, av, P) == oracle.align_prefix(L, hit, av, P)
+
+
+@pytest.mark.parametrize("args", [
+    (0, 0, [], 16), (10, 11, [], 16), (10, -1, [], 16), (10, 5, [], 0),
+    (10, 10, [4, 4], 2), (10, 10, [8, 4], 2), (10, 10, [-4], 2)])
+def test_align_invalid(args):
+    with pytest.raises(hs.HsError) as e:
+        hs.hs_align_prefix(*args)
+    assert e.value.status == hs.HS_ERR_INVALID_ARG
+
+
+def test_num_checkpoints_matches_oracle():
+    rng = np.random.default_rng(5)
+    for _ in range(500):
+        B = int(rng.integers(1, 6))
+        pos0 = rng.integers(0, 5000, size=B)
+        nt = rng.integers(0, 3000, size=B)
+        C = int(rng.choice([0, 64, 256, 512]))
+        want = sum(oracle.n_checkpoints(int(p), int(n), C) for p, n in zip(pos0, nt))
+        assert hs.hs_linattn_num_checkpoints(pos0, nt, C) == want
+
+
+FAKE = 1 << 20        # a 16-byte aligned non-null address that is never dereferenced
+
+
+def test_kv_pages_host_validation():
+    def call(**kw):
+        a = dict(staging_layers=FAKE, cache_layers=FAKE, n_layers=1, block_table=FAKE, n_pages=1,
+                 page_bytes=64, num_blocks=4, d_err=None, stream=0)
+        a.update(kw)
+        hs.hs_restore_kv_pages(**a)
+    for kw, code in [(dict(n_layers=-1), hs.HS_ERR_INVALID_ARG),
+                     (dict(page_bytes=0), hs.HS_ERR_INVALID_ARG),
+                     (dict(page_bytes=24), hs.HS_ERR_MISALIGNED),
+                     (dict(staging_layers=None), hs.HS_ERR_INVALID_ARG),
+                     (dict(block_table=None), hs.HS_ERR_INVALID_ARG),
+                     (dict(n_pages=5, num_blocks=4), hs.HS_ERR_INVALID_ARG)]:
+        with pytest.raises(hs.HsError) as e:
+            call(**kw)
+        assert e.value.status == code, kw
+    call(n_layers=0)          # no-ops return OK without touching the GPU
+    call(n_pages=0)
+
+
+def test_state_copy_host_validation():
+    for fn in (hs.hs_restore_state, hs.hs_checkpoint_states):
+        with pytest.raises(hs.HsError):
+            fn(FAKE, FAKE, -1, 16, stream=0)
+        with pytest.raises(hs.HsError):
+            fn(None, FAKE, 2, 16, stream=0)
+        fn(FAKE, FAKE, 0, 16, stream=0)
+        fn(None, None, 3, 0, stream=0)
+
+
+def test_prefill_host_validation():
+    def call(shape_kw=None, **kw):
+        sk = dict(batch=1, n_heads=2, d_k=64, d_v=64, max_tokens=8)
+        sk.update(shape_kw or {})
+        a = dict(q=FAKE, k=FAKE, v=FAKE, log_g=FAKE, o=FAKE, state=FAKE, pos0=[0], n_tokens=[8],
+                 ckpt_interval=64, ckpt_slots=None, d_err=None, stream=0)
+        a.update(kw)
+        hs.hs_linattn_prefill_from_state(hs.make_shape(**sk), **a)
+    cases = [
+        (dict(shape_kw=dict(d_k=96, d_v=96)), hs.HS_ERR_UNSUPPORTED),
+        (dict(shape_kw=dict(d_k=64, d_v=128)), hs.HS_ERR_UNSUPPORTED),
+        (dict(shape_kw=dict(batch=hs.HS_MAX_BATCH + 1), pos0=[0] * 513, n_tokens=[1] * 513),
+         hs.HS_ERR_UNSUPPORTED),
+        (dict(ckpt_interval=96), hs.HS_ERR_UNSUPPORTED),
+        (dict(ckpt_interval=-64), hs.HS_ERR_INVALID_ARG),
+        (dict(shape_kw=dict(n_heads=0)), hs.HS_ERR_INVALID_ARG),
+        (dict(n_tokens=[9]), hs.HS_ERR_INVALID_ARG),
+        (dict(pos0=[-1]), hs.HS_ERR_INVALID_ARG),
+        (dict(q=None), hs.HS_ERR_INVALID_ARG),
+        (dict(state=None), hs.HS_ERR_INVALID_ARG),
+        (dict(o=FAKE + 4), hs.HS_ERR_MISALIGNED),
+        (dict(log_g=FAKE + 8), hs.HS_ERR_MISALIGNED),
+        (dict(shape_kw=dict(kernel=7)), hs.HS_ERR_INVALID_ARG),
+    ]
+    for kw, code in cases:
+        with pytest.raises(hs.HsError) as e:
+            call(**kw)
+        assert e.value.status == code, kw
+    call(shape_kw=dict(batch=0), pos0=[], n_tokens=[])    # empty batch: OK, nothing launched
+    call(n_tokens=[0], q=None, k=None, v=None, log_g=None, o=None)   # empty tails: OK
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    import importlib
+    mod = importlib.import_module("paper_2609_15030_gb300")
+    monkeypatch.setattr(mod, "LIB_PATH", str(tmp_path / "absent.so"))
+    monkeypatch.setattr(mod, "_lib", None)
+    with pytest.raises(RuntimeError):
+        mod.hs_version()

@@ -1,0 +1,235 @@
+"""Gated linear-attention prefill on the GPU against the float64 oracle.
+
+Parity bar: outputs, final states and checkpoints within a max-normalised
+relative error of 2e-3 per (request, head) tensor; resuming from a
+checkpoint on the absolute chunk grid must reproduce the GPU's own full
+recomputation bit for bit (the paper's matched checkpoint schedule, Section
+4.1 and Table 2), for outputs, final states and emitted checkpoints.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_15030_gb300 as hs
+from hs_inputs import LONG24, SWEEP, TINY, gen_linear, gen_state
+from tests.gpu_helpers import TOL, device, maxnorm_err, run_prefill, to_dev
+
+pytestmark = pytest.mark.gpu
+KERNELS = [hs.HS_LINATTN_RECURRENT]
+
+
+def _check(o, S, cks, ro, rS, rcks, pos0, n_tokens, what=""):
+    for b, n in enumerate(n_tokens):
+        if n:
+            e = maxnorm_err(o[b, :n], ro[b, :n], axes=(0, 2))
+            assert e <= TOL, f"{what} outputs b={b}: {e:.3g}"
+    e = maxnorm_err(S, rS, axes=(2, 3))
+    assert e <= TOL, f"{what} state: {e:.3g}"
+    for b in range(len(n_tokens)):
+        assert cks[b].shape == rcks[b].shape
+        if cks[b].shape[0]:
+            e = maxnorm_err(cks[b], rcks[b], axes=(2, 3))
+            assert e <= TOL, f"{what} checkpoints b={b}: {e:.3g}"
+
+
+def _resume_equals_recompute(inp, N, c, C, dev, kernel):
+    """GPU full recomputation of [0,N) vs GPU resume from its own checkpoint at c."""
+    o_f, S_f, ck_f = run_prefill(inp, [0], [N], None, C, dev, kernel)
+    m = c // C - 1
+    S_c = ck_f[0][m][None] if c > 0 else None
+    sub = type(inp)(*(x[:, c:N].copy() for x in (inp.q, inp.k, inp.v, inp.a)))
+    o_r, S_r, ck_r = run_prefill(sub, [c], [N - c], S_c, C, dev, kernel)
+    assert np.array_equal(o_r[0].view(np.uint32), o_f[0, c:N].view(np.uint32))
+    assert np.array_equal(S_r.view(np.uint32), S_f.view(np.uint32))
+    assert np.array_equal(ck_r[0].view(np.uint32), ck_f[0][m + 1:].view(np.uint32))
+    return o_f, S_f, ck_f
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_tiny_hybrid_config(kernel):
+    """Tiny stack: N=256, C=64, complete hit -> c=192; 64-token tail vs full recompute of 256."""
+    dev = device()
+    N, C = 256, TINY.ckpt
+    c, _, tail = hs.hs_align_prefix(N, N, list(range(C, N + 1, C)), TINY.page)
+    assert (c, tail) == (192, 64)
+    inp = gen_linear(0, 0, 1, N, TINY.n_heads, TINY.d, TINY.d, gates=TINY.gates)
+    o_f, S_f, ck_f = _resume_equals_recompute(inp, N, c, C, dev, kernel)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], C_=C)
+    _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], "tiny")
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("L", [512, 1536, 4608])
+def test_sweep_config_complete_and_partial_hit(kernel, L):
+    """Single-layer sweep: 16 heads, d=128, C=512; complete hit and hit = L-37."""
+    dev = device()
+    C = SWEEP.ckpt
+    inp = gen_linear(1, 0, 1, L, SWEEP.n_heads, SWEEP.d, SWEEP.d, gates=SWEEP.gates)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [L], C_=C, threads=16)
+    for hit in (L, L - 37):
+        c, _, tail = hs.hs_align_prefix(L, hit, list(range(C, L + 1, C)), SWEEP.page)
+        assert tail >= 1 and c % C == 0
+        o_f, S_f, ck_f = _resume_equals_recompute(inp, L, c, C, dev, kernel)
+        _check(o_f, S_f, ck_f, ro, rS, rck, [0], [L], f"L={L} hit={hit}")
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_ragged_prompt_lengths(kernel):
+    """Complete hits at N = L-37 leave a ragged last chunk; several tail lengths."""
+    dev = device()
+    C = 128
+    for N in (1, 3, 63, 65, 130, 475):
+        inp = gen_linear(2, N, 1, N, 4, 128, 128)
+        c, _, _ = hs.hs_align_prefix(N, N, list(range(C, N + 1, C)), 16)
+        o_f, S_f, ck_f = _resume_equals_recompute(inp, N, c, C, dev, kernel)
+        ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], C_=C)
+        _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], f"N={N}")
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+@pytest.mark.parametrize("d", [64, 128])
+def test_batch_mixed_positions_from_nonzero_state(kernel, d):
+    dev = device()
+    B, T, nH = 5, 200, 3
+    pos0 = [0, 64, 128 + 5, 1000, 7]
+    n_tok = [200, 0, 77, 129, 1]
+    inp = gen_linear(3, 0, B, T, nH, d, d)
+    S0 = gen_state(3, 0, B, nH, d, d)
+    o, S, cks = run_prefill(inp, pos0, n_tok, S0, 64, dev, kernel)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, pos0, n_tok, S0=S0, C_=64)
+    _check(o, S, cks, ro, rS, rck, pos0, n_tok, "batch")
+    np.testing.assert_array_equal(S[1], S0[1])          # empty tail leaves the state untouched
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_decode_steps_continue_the_prefill(kernel):
+    """Hybrid workload shape: tail prefill then single-token decode steps off the grid."""
+    dev = device()
+    N, c, steps, nH, d = 512, 256, 16, 16, 128
+    inp = gen_linear(4, 0, 1, N + steps, nH, d, d)
+    ro, rS, _ = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N + steps], threads=16)
+    _, S_c, _ = oracle.gla(inp.q[:, :c], inp.k[:, :c], inp.v[:, :c], inp.a[:, :c], [0], [c],
+                           threads=16)
+    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    state = to_dev(S_c.astype(np.float32), dev)
+    o = torch.zeros((1, N + steps, nH, d), device=dev)
+    T = N + steps
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def call(p0, n):
+        # views starting at token p0; the token extent stays T so strides are unchanged
+        off = p0 * nH * d
+        hs.hs_linattn_prefill_from_state(hs.make_shape(1, nH, d, d, T - p0, kernel),
+                                         q.view(-1)[off:], k.view(-1)[off:], v.view(-1)[off:],
+                                         a.view(-1)[off:], o.view(-1)[off:], state, [p0], [n], 0,
+                                         None, err)
+    call(c, N - c)
+    for s in range(steps):
+        call(N + s, 1)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    got = o.cpu().numpy()
+    assert maxnorm_err(got[0, c:], ro[0, c:], axes=(0, 2)) <= TOL
+    assert maxnorm_err(state.cpu().numpy(), rS, axes=(2, 3)) <= TOL
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_zero_and_identity_gates(kernel):
+    dev = device()
+    N, nH, d = 150, 2, 64
+    for fill in (-1e4, 0.0):
+        inp = gen_linear(5, 0, 1, N, nH, d, d)
+        inp.a[:] = fill
+        S0 = gen_state(5, 0, 1, nH, d, d)
+        o, S, cks = run_prefill(inp, [0], [N], S0, 64, dev, kernel)
+        ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], S0=S0, C_=64)
+        _check(o, S, cks, ro, rS, rck, [0], [N], f"gate={fill}")
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_fused_checkpoints_equal_standalone_writer(kernel):
+    """A prefill ending on a checkpoint boundary: its fused checkpoint equals a
+    snapshot of the live state taken by hs_checkpoint_states, bit for bit."""
+    dev = device()
+    N, C, nH, d = 512, 256, 8, 128
+    inp = gen_linear(6, 0, 1, N, nH, d, d)
+    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    state = torch.zeros((1, nH, d, d), device=dev)
+    o = torch.zeros((1, N, nH, d), device=dev)
+    slots = torch.zeros((2, nH, d, d), device=dev)
+    snap = torch.zeros((nH, d, d), device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_linattn_prefill_from_state(hs.make_shape(1, nH, d, d, N, kernel), q, k, v, a, o, state,
+                                     [0], [N], C, hs.ptr_array([slots[0], slots[1]], dev), err)
+    hs.hs_checkpoint_states(hs.ptr_array([state], dev), hs.ptr_array([snap], dev), 1,
+                            nH * d * d, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    assert torch.equal(slots[1].view(torch.int32), snap.view(torch.int32))
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_checkpoint_slot_errors_are_reported(kernel):
+    dev = device()
+    N, nH, d = 128, 2, 64
+    inp = gen_linear(7, 0, 1, N, nH, d, d)
+    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    state = torch.zeros((1, nH, d, d), device=dev)
+    o = torch.zeros((1, N, nH, d), device=dev)
+    slot = torch.zeros(nH * d * d + 4, device=dev)
+    for ptrs, code in (([slot.data_ptr() + 4, slot.data_ptr()], hs.HS_DEVERR_MISALIGNED),
+                       ([0, slot.data_ptr()], hs.HS_DEVERR_NULL)):
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+        state.zero_()
+        hs.hs_linattn_prefill_from_state(hs.make_shape(1, nH, d, d, N, kernel), q, k, v, a, o,
+                                         state, [0], [N], 64, hs.ptr_array(ptrs, dev), err)
+        torch.cuda.synchronize()
+        assert err.item() == code
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_long_context_full_size_sampled_heads(kernel):
+    """Long-context stack shape at L = 16384: batch 4, 32 heads, d=128, C=512,
+    inputs drawn on the device; sampled (request, head) pairs against the oracle,
+    and the resumed tail (hit = L-37) bitwise against the full recomputation."""
+    dev = device()
+    from hs_inputs import torch_gen_linear
+    L, C, B, nH, d = 16384, LONG24.ckpt, LONG24.batch, LONG24.n_heads, LONG24.d
+    q, k, v, a = torch_gen_linear(11, 0, B, L, nH, d, dev)
+    state = torch.zeros((B, nH, d, d), device=dev)
+    o = torch.zeros((B, L, nH, d), device=dev)
+    nck = hs.hs_linattn_num_checkpoints([0] * B, [L] * B, C)
+    slots = torch.zeros((nck, nH, d, d), device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_linattn_prefill_from_state(hs.make_shape(B, nH, d, d, L, kernel), q, k, v, a, o, state,
+                                     [0] * B, [L] * B, C,
+                                     hs.ptr_array([slots[i] for i in range(nck)], dev), err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    c, _, tail = hs.hs_align_prefix(L, L - 37, list(range(C, L + 1, C)), LONG24.page)
+    per = L // C
+    # resume every request from its checkpoint at c
+    st2 = torch.stack([slots[b * per + c // C - 1] for b in range(B)]).contiguous()
+    o2 = torch.zeros((B, tail, nH, d), device=dev)
+    sl2 = torch.zeros((B, nH, d, d), device=dev)
+    hs.hs_linattn_prefill_from_state(hs.make_shape(B, nH, d, d, tail, kernel),
+                                     q[:, c:].contiguous(), k[:, c:].contiguous(),
+                                     v[:, c:].contiguous(), a[:, c:].contiguous(), o2, st2,
+                                     [c] * B, [tail] * B, C,
+                                     hs.ptr_array([sl2[b] for b in range(B)], dev), err)
+    torch.cuda.synchronize()
+    assert torch.equal(o2.view(torch.int32), o[:, c:].view(torch.int32))
+    assert torch.equal(st2.view(torch.int32), state.view(torch.int32))
+    assert torch.equal(sl2.view(torch.int32), slots[per - 1::per].view(torch.int32))
+    # sampled heads against the oracle (float64, token by token)
+    for b, h in ((0, 0), (3, 31)):
+        qh = q[b:b + 1, :, h:h + 1].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        kh = k[b:b + 1, :, h:h + 1].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        vh = v[b:b + 1, :, h:h + 1].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        ah = a[b:b + 1, :, h:h + 1].contiguous().cpu().numpy()
+        ro, rS, rck = oracle.gla(qh, kh, vh, ah, [0], [L], C_=C)
+        assert maxnorm_err(o[b, :, h].cpu().numpy(), ro[0, :, 0], axes=(0, 1)) <= TOL
+        assert maxnorm_err(state[b, h].cpu().numpy(), rS[0, 0], axes=(0, 1)) <= TOL
+        got_ck = slots[b * per:(b + 1) * per, h].cpu().numpy()
+        assert maxnorm_err(got_ck, rck[0][:, 0], axes=(1, 2)) <= TOL
