@@ -151,9 +151,12 @@ hs_status hs_checkpoint_states(const float *const *live_states, float *const *ck
 
 /* Which kernel hs_linattn_prefill_from_state runs. */
 typedef enum hs_linattn_kernel {
-    HS_LINATTN_AUTO = 0,       /* the library's choice for the shape */
+    HS_LINATTN_AUTO = 0,       /* chunked tensor-core kernel when d_k == d_v == 128 and
+                                  batch*max_tokens < 2^31, else the recurrent kernel; the
+                                  choice depends on the shape only */
     HS_LINATTN_RECURRENT = 1,  /* per-token recurrence, CUDA cores */
-    HS_LINATTN_CHUNKED_TC = 2  /* chunked form on tcgen05 tensor cores */
+    HS_LINATTN_CHUNKED_TC = 2  /* chunked form on tcgen05 tensor cores (d_k == d_v == 128;
+                                  HS_ERR_UNSUPPORTED otherwise) */
 } hs_linattn_kernel;
 
 typedef struct hs_linattn_shape {

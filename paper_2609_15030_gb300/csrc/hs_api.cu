@@ -225,7 +225,13 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
     if (base > INT32_MAX)
         return HS_ERR_INVALID_ARG;
 
-    if (s.kernel == HS_LINATTN_CHUNKED_TC)
+    const bool tc_ok = hs::gla_chunked_tc_supported(s.d_k, s.batch, s.max_tokens);
+    if (s.kernel == HS_LINATTN_CHUNKED_TC && !tc_ok)
+        return HS_ERR_UNSUPPORTED;
+    // AUTO depends on the shape only (never on positions or token counts), so two
+    // runs with the same shape always take the same kernel
+    const bool use_tc = s.kernel == HS_LINATTN_CHUNKED_TC || (s.kernel == HS_LINATTN_AUTO && tc_ok);
+    if (use_tc)
         return cuda_status(hs::launch_gla_chunked_tc(p, s.d_k, stream));
     return cuda_status(hs::launch_gla_recurrent(p, s.d_k, stream));
 }

@@ -43,5 +43,6 @@ cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t
                              int64_t floats_each, int32_t *d_err, int sm_count, cudaStream_t s);
 cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s);
+bool gla_chunked_tc_supported(int d, int64_t batch, int64_t max_tokens);
 
 }  // namespace hs

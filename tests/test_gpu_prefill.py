@@ -16,7 +16,14 @@ from hs_inputs import LONG24, SWEEP, TINY, gen_linear, gen_state
 from tests.gpu_helpers import TOL, device, maxnorm_err, run_prefill, to_dev
 
 pytestmark = pytest.mark.gpu
-KERNELS = [hs.HS_LINATTN_RECURRENT]
+KERNELS = [pytest.param(hs.HS_LINATTN_RECURRENT, id="recurrent"),
+           pytest.param(hs.HS_LINATTN_CHUNKED_TC, id="tc")]
+
+
+def _needs(kernel, d):
+    """The tensor-core kernel implements d = 128 only (HS_ERR_UNSUPPORTED otherwise)."""
+    if kernel == hs.HS_LINATTN_CHUNKED_TC and d != 128:
+        pytest.skip("chunked tensor-core kernel: d = 128 only")
 
 
 def _check(o, S, cks, ro, rS, rcks, pos0, n_tokens, what=""):
@@ -49,6 +56,7 @@ def _resume_equals_recompute(inp, N, c, C, dev, kernel):
 @pytest.mark.parametrize("kernel", KERNELS)
 def test_tiny_hybrid_config(kernel):
     """Tiny stack: N=256, C=64, complete hit -> c=192; 64-token tail vs full recompute of 256."""
+    _needs(kernel, TINY.d)
     dev = device()
     N, C = 256, TINY.ckpt
     c, _, tail = hs.hs_align_prefix(N, N, list(range(C, N + 1, C)), TINY.page)
@@ -90,6 +98,7 @@ def test_ragged_prompt_lengths(kernel):
 @pytest.mark.parametrize("kernel", KERNELS)
 @pytest.mark.parametrize("d", [64, 128])
 def test_batch_mixed_positions_from_nonzero_state(kernel, d):
+    _needs(kernel, d)
     dev = device()
     B, T, nH = 5, 200, 3
     pos0 = [0, 64, 128 + 5, 1000, 7]
@@ -100,6 +109,23 @@ def test_batch_mixed_positions_from_nonzero_state(kernel, d):
     ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, pos0, n_tok, S0=S0, C_=64)
     _check(o, S, cks, ro, rS, rck, pos0, n_tok, "batch")
     np.testing.assert_array_equal(S[1], S0[1])          # empty tail leaves the state untouched
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_mixed_gate_strengths_take_both_paths(kernel):
+    """Chunks whose per-dimension decay exceeds 2^-64 (the tensor-core kernel's
+    exact path) interleaved with ordinary chunks; both must match the oracle and
+    keep resume == recompute bitwise."""
+    dev = device()
+    N, C, nH, d = 448, 64, 4, 128
+    inp = gen_linear(12, 0, 1, N, nH, d, d)
+    inp.a[:, 70:75, :, :7] = -30.0          # strong decay on a few key dims in chunk 1
+    inp.a[:, 200, 1] = -1e4                 # a zero gate for head 1 in chunk 3
+    inp.a[:, 300:364, 2] = -1.2             # steady strong decay over a whole chunk
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], C_=C)
+    for c in (64, 192, 320):
+        o_f, S_f, ck_f = _resume_equals_recompute(inp, N, c, C, dev, kernel)
+    _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], "mixed gates")
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
@@ -135,9 +161,11 @@ def test_decode_steps_continue_the_prefill(kernel):
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
-def test_zero_and_identity_gates(kernel):
+@pytest.mark.parametrize("d", [64, 128])
+def test_zero_and_identity_gates(kernel, d):
+    _needs(kernel, d)
     dev = device()
-    N, nH, d = 150, 2, 64
+    N, nH = 150, 2
     for fill in (-1e4, 0.0):
         inp = gen_linear(5, 0, 1, N, nH, d, d)
         inp.a[:] = fill
@@ -172,7 +200,7 @@ def test_fused_checkpoints_equal_standalone_writer(kernel):
 @pytest.mark.parametrize("kernel", KERNELS)
 def test_checkpoint_slot_errors_are_reported(kernel):
     dev = device()
-    N, nH, d = 128, 2, 64
+    N, nH, d = 128, 2, 128
     inp = gen_linear(7, 0, 1, N, nH, d, d)
     q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
     state = torch.zeros((1, nH, d, d), device=dev)
