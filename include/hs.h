@@ -62,6 +62,9 @@ typedef enum hs_status {
 #define HS_MAX_BATCH 512
 /* Chunk length of the prefill; checkpoint intervals are multiples of it. */
 #define HS_CHUNK 64
+/* Segments (the part of a call inside one chunk) of at most this many tokens are
+ * computed token by token, with the same arithmetic in every kernel. */
+#define HS_SHORT_SEGMENT 8
 
 /* Human-readable name of a status; never NULL. */
 const char *hs_status_string(hs_status s);
@@ -151,9 +154,10 @@ hs_status hs_checkpoint_states(const float *const *live_states, float *const *ck
 
 /* Which kernel hs_linattn_prefill_from_state runs. */
 typedef enum hs_linattn_kernel {
-    HS_LINATTN_AUTO = 0,       /* chunked tensor-core kernel when d_k == d_v == 128 and
-                                  batch*max_tokens < 2^31, else the recurrent kernel; the
-                                  choice depends on the shape only */
+    HS_LINATTN_AUTO = 0,       /* chunked tensor-core kernel when d_k == d_v == 128,
+                                  batch*max_tokens < 2^31 and some n_tokens exceeds
+                                  HS_SHORT_SEGMENT; else the recurrent kernel.  Both compute
+                                  short segments identically, so AUTO never changes results */
     HS_LINATTN_RECURRENT = 1,  /* per-token recurrence, CUDA cores */
     HS_LINATTN_CHUNKED_TC = 2  /* chunked form on tcgen05 tensor cores (d_k == d_v == 128;
                                   HS_ERR_UNSUPPORTED otherwise) */
@@ -183,10 +187,11 @@ typedef struct hs_linattn_shape {
  *
  * For problem b, token t < n_tokens[b] of q/k/v/log_g/o is absolute position
  * pos0[b] + t.  state[b] holds on entry the state of prefix [0,pos0[b]) and on
- * return that of [0,pos0[b]+n_tokens[b]).  Work is split into chunks of
- * HS_CHUNK tokens on the absolute position grid and every chunk is a fixed
- * function of its inputs and its incoming state, so resuming at a multiple of
- * HS_CHUNK reproduces a full recomputation bit for bit (same kernel choice).
+ * return that of [0,pos0[b]+n_tokens[b]).  Work is split into segments at the
+ * multiples of HS_CHUNK on the absolute position grid and every segment is a
+ * fixed function of its inputs and its incoming state, so resuming at a
+ * multiple of HS_CHUNK reproduces a full recomputation bit for bit (with AUTO,
+ * or with the same explicit kernel in both runs).
  *
  *   shp        host; batch in [0, HS_MAX_BATCH]; d_k == d_v in {64,128}
  *   q, k       device bf16 [batch][max_tokens][n_heads][d_k]

@@ -33,6 +33,7 @@ HS_DEVERR_TIMEOUT = 4
 
 HS_MAX_BATCH = 512
 HS_CHUNK = 64
+HS_SHORT_SEGMENT = 8
 
 HS_LINATTN_AUTO = 0
 HS_LINATTN_RECURRENT = 1

@@ -55,6 +55,7 @@ using namespace ptx;
 constexpr int D = 128;    // d_k = d_v
 constexpr int CH = 64;    // chunk length (absolute grid)
 constexpr int NT = 256;   // threads per CTA
+constexpr int kShort = 8; // segments of at most this many tokens run token by token
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kFastMinLog2 = -64.0f;      // factorised form if every 2^{Lam_last} >= 2^-64
 constexpr uint64_t kTimeoutNs = 1000000000ull;
@@ -94,13 +95,13 @@ struct TmaMaps {
 // Byte offset of element (row, col) of a row-major f32 operand stored as
 // 32-column slabs (128-byte rows) in the 128-byte swizzled K-major canonical
 // layout: 16-byte chunk c of row r sits at chunk position c ^ (r % 8).
-// sw_off: 64-row operands; sw_off_t: 128-row operands.
 __device__ __forceinline__ uint32_t sw_off(int row, int col)
 {
     return (uint32_t)((col >> 5) * SLAB + row * 128 + ((((col & 31) >> 2) ^ (row & 7)) << 4) +
                       ((col & 3) << 2));
 }
 
+// 16-byte chunk col4 (columns 4*col4 .. 4*col4+3) of row `row` of a 128-row operand
 __device__ __forceinline__ uint32_t sw_chunk_t(int row, int col4)
 {
     return (uint32_t)((col4 >> 3) * SLAB_T + row * 128 + (((col4 & 7) ^ (row & 7)) << 4));
@@ -109,6 +110,30 @@ __device__ __forceinline__ uint32_t sw_chunk_t(int row, int col4)
 __device__ __forceinline__ float bf16f(uint16_t x)
 {
     return __uint_as_float(((uint32_t)x) << 16);
+}
+
+__device__ __forceinline__ float bf_lo(uint32_t w)
+{
+    return __uint_as_float(w << 16);
+}
+
+__device__ __forceinline__ float bf_hi(uint32_t w)
+{
+    return __uint_as_float(w & 0xFFFF0000u);
+}
+
+// 2^x, one MUFU op (relative error ~2^-22; inputs here lie in [-2^7, 2^7])
+__device__ __forceinline__ float ex2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// round to tf32 (nearest, ties away from zero) with integer ops; low 13 bits cleared
+__device__ __forceinline__ float rna_tf32(float x)
+{
+    return __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
 }
 
 __global__ void __launch_bounds__(NT, 1)
@@ -186,6 +211,25 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
         tmem_wait_st();
     }
+
+    // operand-building map: thread owns key dims (dp, dp+1) of tokens [16*qr, 16*qr+16)
+    const int qr = lane >> 3;
+    const int dp = 2 * (warp * 8 + (lane & 7));
+    uint32_t nat[8];       // byte offset of (row 16*qr + r, col dp) in a 64-row operand
+    {
+        const uint32_t base = (uint32_t)((dp >> 5) * SLAB + (16 * qr) * 128 + ((dp & 3) << 2));
+        const int cd = (dp & 31) >> 2;
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+            nat[r] = base + r * 128 + ((uint32_t)(cd ^ r) << 4);
+    }
+    uint32_t tr0[4], tr1[4];   // 16-byte chunk (tokens 16*qr + 4g ..) of rows dp, dp+1 of a 128-row operand
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+        tr0[g] = sw_chunk_t(dp, 4 * qr + g);
+        tr1[g] = sw_chunk_t(dp + 1, 4 * qr + g);
+    }
+
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -197,7 +241,17 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         const int64_t seg_end = min(end, (pos / CH + 1) * CH);
         const int L = (int)(seg_end - pos);
         const bool has_next = seg_end < end;
-        const bool ckpt = (C > 0) && (seg_end % C == 0);
+        float *slot = nullptr;     // checkpoint slot of this segment's end, if any
+        if (C > 0 && seg_end % C == 0 && p.ckpt_slots != nullptr) {
+            slot = p.ckpt_slots[p.ck_base[b] + (seg_end / C - pos0 / C - 1)];
+            if (slot == nullptr || (reinterpret_cast<uintptr_t>(slot) & 15u) != 0) {
+                if (tid == 0)
+                    report(p.d_err, slot == nullptr ? HS_DEVERR_NULL : HS_DEVERR_MISALIGNED);
+                slot = nullptr;
+            } else {
+                slot += (int64_t)h * D * D;
+            }
+        }
 
         // ---- 1. staged inputs
         if (tid == 0) {
@@ -213,58 +267,178 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
         ph_tma ^= 1;
 
-        // ---- 2. operands: thread (d, half) scans tokens [32*half, 32*half+32) of key dim d
-        const int d = 16 * warp + (lane & 15);
-        const int half = lane >> 4;
-        const int i0 = half * 32;
-        float lam[32];
-        float run = 0.f;
+        if (L <= kShort) {
+            // ---- short segment: the per-token recurrence, with the recurrent kernel's
+            // exact operation order (two 64-row halves of each state column, each a
+            // sequential fma chain; o = half0 + half1), so both kernels agree bit for bit
+            for (int idx = tid; idx < L * D; idx += NT)
+                sG[idx] = expf(sG[idx]);
+            __syncthreads();
+            float S[64];
+            tmem_ld32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
+            tmem_ld32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
+            tmem_wait_ld();
+            float *part = reinterpret_cast<float *>(smem + OFF_A);   // [kShort][2][128]
+            for (int i = 0; i < L; ++i) {
+                const float ve = bf16f(sV[i * D + e_own]);
+                float acc = 0.f;
 #pragma unroll
-        for (int x = 0; x < 32; ++x) {
-            const int i = i0 + x;
-            const float a = (i < L) ? sG[i * D + d] : 0.f;
-            run = fmaf(a, kLog2e, run);
-            lam[x] = run;
-        }
-        const float tot_lo = __shfl_sync(0xffffffffu, run, lane & 15);
-        const float tot_hi = __shfl_sync(0xffffffffu, run, (lane & 15) + 16);
-        if (half) {
-#pragma unroll
-            for (int x = 0; x < 32; ++x)
-                lam[x] = tot_lo + lam[x];
-        }
-        const float lam_last = tot_lo + tot_hi;
-        if (half == 0)
-            sGam[d] = exp2f(lam_last);
-        const bool slow = __syncthreads_or(lam_last < kFastMinLog2) != 0;
-
-#pragma unroll
-        for (int x4 = 0; x4 < 32; x4 += 4) {
-            float4 kt4, vt4;
-            float *ktv = reinterpret_cast<float *>(&kt4), *vtv = reinterpret_cast<float *>(&vt4);
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int x = x4 + u;
-                const int i = i0 + x;
-                const bool valid = i < L;
-                const float qv = valid ? bf16f(sQ[i * D + d]) : 0.f;
-                const float kv = valid ? bf16f(sK[i * D + d]) : 0.f;
-                const float l = lam[x];
-                const uint32_t o = sw_off(i, d);
-                *reinterpret_cast<float *>(smem + OFF_QT + o) = to_tf32(qv * exp2f(l));
-                if (slow) {
-                    ktv[u] = to_tf32(kv * exp2f(lam_last - l));   // K^ = k 2^{Lam_last - Lam}
-                    sG[i * D + d] = l;    // cumulative log2-gates, in place, for the exact path
-                } else {
-                    const float kt = to_tf32(kv * exp2f(-l));
-                    *reinterpret_cast<float *>(smem + OFF_KT + o) = kt;
-                    ktv[u] = kt;
+                for (int r = 0; r < 64; ++r) {
+                    const int d = colhalf * 64 + r;
+                    S[r] = fmaf(sG[i * D + d], S[r], bf16f(sK[i * D + d]) * ve);
+                    acc = fmaf(bf16f(sQ[i * D + d]), S[r], acc);
                 }
-                vtv[u] = valid ? bf16f(sV[i * D + d]) : 0.f;
+                part[(i * 2 + colhalf) * D + e_own] = acc;
             }
-            const uint32_t ot = sw_chunk_t(d, (i0 + x4) >> 2);
-            *reinterpret_cast<float4 *>(smem + OFF_KTT + ot) = kt4;
-            *reinterpret_cast<float4 *>(smem + OFF_VT + ot) = vt4;
+            tmem_st32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
+            tmem_st32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
+            if (slot != nullptr) {
+#pragma unroll
+                for (int r = 0; r < 64; ++r)
+                    slot[(int64_t)(colhalf * 64 + r) * D + e_own] = S[r];
+            }
+            tmem_wait_st();
+            fence_proxy_async_smem();
+            __syncthreads();
+            if (tid == 0 && has_next)
+                issue_tma(tok + L);
+            float *ob = p.o + (((int64_t)b * p.max_tokens + tok) * p.n_heads + h) * D;
+            for (int idx = tid; idx < L * D; idx += NT) {
+                const int i = idx >> 7, e = idx & (D - 1);
+                ob[(int64_t)i * tstride + e] = part[(i * 2) * D + e] + part[(i * 2 + 1) * D + e];
+            }
+            tc_fence_before();
+            __syncthreads();
+            tc_fence_after();
+            pos = seg_end;
+            tok += L;
+            continue;
+        }
+
+        if (L < CH) {
+            // zero the staged rows past the segment: every operand row >= L becomes 0
+            for (int idx = tid; idx < (CH - L) * 80; idx += NT) {
+                const int row = L + idx / 80, c = idx % 80;
+                uint4 *dst;
+                if (c < 16)
+                    dst = reinterpret_cast<uint4 *>(smem + OFF_SQ + row * 256) + c;
+                else if (c < 32)
+                    dst = reinterpret_cast<uint4 *>(smem + OFF_SK + row * 256) + (c - 16);
+                else if (c < 48)
+                    dst = reinterpret_cast<uint4 *>(smem + OFF_SV + row * 256) + (c - 32);
+                else
+                    dst = reinterpret_cast<uint4 *>(smem + OFF_SG + row * 512) + (c - 48);
+                *dst = make_uint4(0u, 0u, 0u, 0u);
+            }
+            __syncthreads();
+        }
+
+        // ---- 2. cumulative log2-gates: 16 tokens per thread, then a shuffle scan
+        //         over the four token quarters that hold the same key dims
+        float lam0[16], lam1[16];
+        float run0 = 0.f, run1 = 0.f;
+#pragma unroll
+        for (int x = 0; x < 16; ++x) {
+            const float2 a2 = *reinterpret_cast<const float2 *>(sG + (16 * qr + x) * D + dp);
+            run0 = fmaf(a2.x, kLog2e, run0);
+            run1 = fmaf(a2.y, kLog2e, run1);
+            lam0[x] = run0;
+            lam1[x] = run1;
+        }
+        float s0 = run0, s1 = run1;
+        {
+            const float y0 = __shfl_up_sync(0xffffffffu, s0, 8);
+            const float y1 = __shfl_up_sync(0xffffffffu, s1, 8);
+            if (qr >= 1) {
+                s0 = s0 + y0;
+                s1 = s1 + y1;
+            }
+        }
+        {
+            const float y0 = __shfl_up_sync(0xffffffffu, s0, 16);
+            const float y1 = __shfl_up_sync(0xffffffffu, s1, 16);
+            if (qr >= 2) {
+                s0 = s0 + y0;
+                s1 = s1 + y1;
+            }
+        }
+        const float pre0 = __shfl_up_sync(0xffffffffu, s0, 8);   // tokens before this quarter
+        const float pre1 = __shfl_up_sync(0xffffffffu, s1, 8);
+        const float last0 = __shfl_sync(0xffffffffu, s0, (lane & 7) + 24);
+        const float last1 = __shfl_sync(0xffffffffu, s1, (lane & 7) + 24);
+        if (qr >= 1) {
+#pragma unroll
+            for (int x = 0; x < 16; ++x) {
+                lam0[x] = pre0 + lam0[x];
+                lam1[x] = pre1 + lam1[x];
+            }
+        }
+        if (qr == 0)
+            *reinterpret_cast<float2 *>(sGam + dp) = make_float2(ex2(last0), ex2(last1));
+        const bool slow = __syncthreads_or(last0 < kFastMinLog2 || last1 < kFastMinLog2) != 0;
+
+        // ---- operands (tf32, K-major, swizzled)
+        if (!slow) {
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+                float4 kt0, kt1, vt0, vt1;
+                float *k0 = &kt0.x, *k1 = &kt1.x, *v0 = &vt0.x, *v1 = &vt1.x;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int x = 4 * g + u;
+                    const int i = 16 * qr + x;
+                    const uint32_t q2 = *reinterpret_cast<const uint32_t *>(sQ + i * D + dp);
+                    const uint32_t k2 = *reinterpret_cast<const uint32_t *>(sK + i * D + dp);
+                    const uint32_t v2 = *reinterpret_cast<const uint32_t *>(sV + i * D + dp);
+                    const uint32_t off = nat[x & 7] + (x >> 3) * 1024;
+                    *reinterpret_cast<float2 *>(smem + OFF_QT + off) =
+                        make_float2(rna_tf32(bf_lo(q2) * ex2(lam0[x])), rna_tf32(bf_hi(q2) * ex2(lam1[x])));
+                    const float ka = rna_tf32(bf_lo(k2) * ex2(-lam0[x]));
+                    const float kb = rna_tf32(bf_hi(k2) * ex2(-lam1[x]));
+                    *reinterpret_cast<float2 *>(smem + OFF_KT + off) = make_float2(ka, kb);
+                    k0[u] = ka;
+                    k1[u] = kb;
+                    v0[u] = bf_lo(v2);
+                    v1[u] = bf_hi(v2);
+                }
+                *reinterpret_cast<float4 *>(smem + OFF_KTT + tr0[g]) = kt0;
+                *reinterpret_cast<float4 *>(smem + OFF_KTT + tr1[g]) = kt1;
+                *reinterpret_cast<float4 *>(smem + OFF_VT + tr0[g]) = vt0;
+                *reinterpret_cast<float4 *>(smem + OFF_VT + tr1[g]) = vt1;
+            }
+        } else {
+#pragma unroll 1
+            for (int g = 0; g < 4; ++g) {
+                float4 kt0, kt1, vt0, vt1;
+                float *k0 = &kt0.x, *k1 = &kt1.x, *v0 = &vt0.x, *v1 = &vt1.x;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int x = 4 * g + u;
+                    const int i = 16 * qr + x;
+                    float la, lb;
+                    // dynamic index into lam (exact path only)
+#pragma unroll
+                    for (int z = 0; z < 16; ++z)
+                        if (z == x) {
+                            la = lam0[z];
+                            lb = lam1[z];
+                        }
+                    const uint32_t q2 = *reinterpret_cast<const uint32_t *>(sQ + i * D + dp);
+                    const uint32_t k2 = *reinterpret_cast<const uint32_t *>(sK + i * D + dp);
+                    const uint32_t v2 = *reinterpret_cast<const uint32_t *>(sV + i * D + dp);
+                    *reinterpret_cast<float2 *>(smem + OFF_QT + sw_off(i, dp)) =
+                        make_float2(rna_tf32(bf_lo(q2) * ex2(la)), rna_tf32(bf_hi(q2) * ex2(lb)));
+                    k0[u] = rna_tf32(bf_lo(k2) * ex2(last0 - la));   // K^ = k 2^{Lam_last - Lam}
+                    k1[u] = rna_tf32(bf_hi(k2) * ex2(last1 - lb));
+                    v0[u] = bf_lo(v2);
+                    v1[u] = bf_hi(v2);
+                    *reinterpret_cast<float2 *>(sG + i * D + dp) = make_float2(la, lb);
+                }
+                *reinterpret_cast<float4 *>(smem + OFF_KTT + sw_chunk_t(dp, 4 * qr + g)) = kt0;
+                *reinterpret_cast<float4 *>(smem + OFF_KTT + sw_chunk_t(dp + 1, 4 * qr + g)) = kt1;
+                *reinterpret_cast<float4 *>(smem + OFF_VT + sw_chunk_t(dp, 4 * qr + g)) = vt0;
+                *reinterpret_cast<float4 *>(smem + OFF_VT + sw_chunk_t(dp + 1, 4 * qr + g)) = vt1;
+            }
         }
         fence_proxy_async_smem();
         __syncthreads();
@@ -291,7 +465,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 issue_tma(tok + L);
         }
 
-        // ---- 3b. the masked intra-chunk matrix A -> shared memory (tf32, K-major)
+        // ---- 3b. the causally masked intra-chunk matrix A -> shared memory
         if (!slow) {
             if (tid == 0 && !mbar_wait_bounded(bar_a, ph_a, kTimeoutNs))
                 sMisc[1] = 1;
@@ -302,22 +476,20 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             ph_a ^= 1;
             tc_fence_after();
-            if (warp < 2) {
-                const int i = warp * 32 + lane;      // TMEM lane = query row
-                float r[2][32];
-                tmem_ld32(tmem + lrow + TM_A, r[0]);
-                tmem_ld32(tmem + lrow + TM_A + 32, r[1]);
+            if ((warp & 3) < 2) {
+                const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
+                const int jb = (warp >> 2) * 32;            // this warp's 32 key columns
+                float r[32];
+                tmem_ld32(tmem + lrow + TM_A + jb, r);
                 tmem_wait_ld();
 #pragma unroll
-                for (int c = 0; c < 16; ++c) {
+                for (int c = 0; c < 8; ++c) {
                     float4 w;
-                    float *wv = reinterpret_cast<float *>(&w);
+                    float *wv = &w.x;
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int j = 4 * c + u;
-                        wv[u] = (j <= i && i < L) ? to_tf32(r[j >> 5][j & 31]) : 0.f;
-                    }
-                    const uint32_t o = (c >> 3) * SLAB + i * 128 + (((c & 7) ^ (i & 7)) << 4);
+                    for (int u = 0; u < 4; ++u)
+                        wv[u] = (jb + 4 * c + u <= i) ? rna_tf32(r[4 * c + u]) : 0.f;
+                    const uint32_t o = (jb >> 5) * SLAB + i * 128 + ((uint32_t)(c ^ (i & 7)) << 4);
                     *reinterpret_cast<float4 *>(smem + OFF_A + o) = w;
                 }
             }
@@ -329,9 +501,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 if (j <= i && i < L) {
                     for (int dd = 0; dd < D; ++dd)
                         acc = fmaf(bf16f(sQ[i * D + dd]) * bf16f(sK[j * D + dd]),
-                                   exp2f(sG[i * D + dd] - sG[j * D + dd]), acc);
+                                   ex2(sG[i * D + dd] - sG[j * D + dd]), acc);
                 }
-                *reinterpret_cast<float *>(smem + OFF_A + sw_off(i, j)) = to_tf32(acc);
+                *reinterpret_cast<float *>(smem + OFF_A + sw_off(i, j)) = rna_tf32(acc);
             }
         }
         fence_proxy_async_smem();
@@ -375,26 +547,20 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             const int ib = colhalf * 32;
             tmem_ld32(tmem + lrow + TM_O + ib, r);
             tmem_wait_ld();
-            float *op = p.o + (((int64_t)b * p.max_tokens + tok) * p.n_heads + h) * D + e_own;
+            float *op = p.o + (((int64_t)b * p.max_tokens + tok + ib) * p.n_heads + h) * D + e_own;
+            if (L == CH) {
 #pragma unroll
-            for (int x = 0; x < 32; ++x)
-                if (ib + x < L)
-                    __stcs(op + (int64_t)(ib + x) * tstride, r[x]);
+                for (int x = 0; x < 32; ++x)
+                    __stcs(op + (int64_t)x * tstride, r[x]);
+            } else {
+#pragma unroll
+                for (int x = 0; x < 32; ++x)
+                    if (ib + x < L)
+                        __stcs(op + (int64_t)x * tstride, r[x]);
+            }
         }
 
         // ---- 4b. state decay (after the update on the factorised path, before it on the exact path)
-        float *slot = nullptr;
-        if (ckpt && p.ckpt_slots != nullptr) {
-            const int64_t idx = p.ck_base[b] + (seg_end / C - pos0 / C - 1);
-            slot = p.ckpt_slots[idx];
-            if (slot == nullptr || (reinterpret_cast<uintptr_t>(slot) & 15u) != 0) {
-                if (tid == 0)
-                    report(p.d_err, slot == nullptr ? HS_DEVERR_NULL : HS_DEVERR_MISALIGNED);
-                slot = nullptr;
-            } else {
-                slot += (int64_t)h * D * D;
-            }
-        }
 #pragma unroll
         for (int c0 = 0; c0 < 64; c0 += 32) {
             const int d0 = colhalf * 64 + c0;
@@ -402,8 +568,13 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             tmem_ld32(tmem + lrow + TM_S + d0, r);
             tmem_wait_ld();
 #pragma unroll
-            for (int x = 0; x < 32; ++x)
-                r[x] *= sGam[d0 + x];
+            for (int c = 0; c < 8; ++c) {
+                const float4 g4 = *reinterpret_cast<const float4 *>(sGam + d0 + 4 * c);
+                r[4 * c] *= g4.x;
+                r[4 * c + 1] *= g4.y;
+                r[4 * c + 2] *= g4.z;
+                r[4 * c + 3] *= g4.w;
+            }
             tmem_st32(tmem + lrow + TM_S + d0, r);
             if (!slow && slot != nullptr) {
 #pragma unroll

@@ -7,6 +7,10 @@
 // registers for the whole call: thread (row group rg, column j) holds rows
 // [rg*R, rg*R+R) of column j.  Tokens are staged eight at a time in shared
 // memory; o_t is the fixed-order sum of the row groups' partial dot products.
+// Per token and element: g = expf(a), S = fmaf(g, S, k*v), partial =
+// fmaf(q, S, partial) in increasing row order; o = partial_0 + partial_1 + ...
+// The chunked tensor-core kernel runs short segments with exactly these
+// operations (d = 128), so the two kernels agree bit for bit on them.
 // The operation order per token depends only on the token's inputs and the
 // incoming state, so resuming from any checkpoint reproduces a full
 // recomputation bit for bit.
@@ -92,9 +96,9 @@ __global__ void __launch_bounds__(kThreads) gla_recurrent_kernel(const __grid_co
         __syncthreads();
         for (int idx = tid; idx < tb * D; idx += kThreads) {
             const int tt = idx / D, e = idx - (idx / D) * D;
-            float s = 0.f;
+            float s = spart[tt][0][e];
 #pragma unroll
-            for (int g = 0; g < NG; ++g)
+            for (int g = 1; g < NG; ++g)
                 s += spart[tt][g][e];
             const int64_t row = ((int64_t)b * p.max_tokens + t0 + tt) * p.n_heads + h;
             p.o[row * D + e] = s;

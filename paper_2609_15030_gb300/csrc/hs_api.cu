@@ -228,9 +228,14 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
     const bool tc_ok = hs::gla_chunked_tc_supported(s.d_k, s.batch, s.max_tokens);
     if (s.kernel == HS_LINATTN_CHUNKED_TC && !tc_ok)
         return HS_ERR_UNSUPPORTED;
-    // AUTO depends on the shape only (never on positions or token counts), so two
-    // runs with the same shape always take the same kernel
-    const bool use_tc = s.kernel == HS_LINATTN_CHUNKED_TC || (s.kernel == HS_LINATTN_AUTO && tc_ok);
+    // AUTO: calls whose tails are all short (decode steps) go to the recurrent kernel,
+    // which computes such segments bit for bit like the chunked kernel does, so the
+    // choice never changes results; everything else takes the tensor-core kernel
+    int32_t max_n = 0;
+    for (int32_t b = 0; b < s.batch; ++b)
+        max_n = n_tokens[b] > max_n ? n_tokens[b] : max_n;
+    const bool use_tc = s.kernel == HS_LINATTN_CHUNKED_TC ||
+                        (s.kernel == HS_LINATTN_AUTO && tc_ok && max_n > HS_SHORT_SEGMENT);
     if (use_tc)
         return cuda_status(hs::launch_gla_chunked_tc(p, s.d_k, stream));
     return cuda_status(hs::launch_gla_recurrent(p, s.d_k, stream));

@@ -261,3 +261,38 @@ def test_long_context_full_size_sampled_heads(kernel):
         assert maxnorm_err(state[b, h].cpu().numpy(), rS[0, 0], axes=(0, 1)) <= TOL
         got_ck = slots[b * per:(b + 1) * per, h].cpu().numpy()
         assert maxnorm_err(got_ck, rck[0][:, 0], axes=(1, 2)) <= TOL
+
+
+def test_short_segments_match_across_kernels():
+    """Calls whose tails are at most HS_SHORT_SEGMENT tokens: the tensor-core
+    kernel's token-by-token path and the recurrent kernel agree bit for bit, so
+    AUTO may send decode steps to either without changing results."""
+    dev = device()
+    B, nH, d, T = 6, 4, 128, 8
+    pos0 = [0, 5, 63, 64, 1000, 4095]
+    n_tok = [8, 1, 2, 7, 3, 8]                       # some straddle a chunk boundary
+    inp = gen_linear(13, 0, B, T, nH, d, d)
+    S0 = gen_state(13, 0, B, nH, d, d)
+    res = [run_prefill(inp, pos0, n_tok, S0, 64, dev, k)
+           for k in (hs.HS_LINATTN_RECURRENT, hs.HS_LINATTN_CHUNKED_TC, hs.HS_LINATTN_AUTO)]
+    for o, S, cks in res[1:]:
+        for b, n in enumerate(n_tok):
+            assert np.array_equal(o[b, :n].view(np.uint32), res[0][0][b, :n].view(np.uint32))
+            assert np.array_equal(cks[b].view(np.uint32), res[0][2][b].view(np.uint32))
+        assert np.array_equal(S.view(np.uint32), res[0][1].view(np.uint32))
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, pos0, n_tok, S0=S0, C_=64)
+    _check(*res[0], ro, rS, rck, pos0, n_tok, "short")
+
+
+@pytest.mark.parametrize("suffix", [1, 3, 4, 5, 8, 9, 64, 65, 127])
+def test_table4_suffix_lengths_auto_resume_bitwise(suffix):
+    """The repaired path recomputes suffixes of 1, 3, 4, 5 and 1,791-1,792 tokens
+    (the paper's Table 4); with the default kernel choice a resumed tail of any
+    length reproduces the full recomputation bit for bit."""
+    dev = device()
+    C, c, nH, d = 128, 256, 4, 128
+    N = c + suffix
+    inp = gen_linear(14, suffix, 1, N, nH, d, d)
+    o_f, S_f, ck_f, = _resume_equals_recompute(inp, N, c, C, dev, hs.HS_LINATTN_AUTO)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], C_=C)
+    _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], f"suffix={suffix}")
