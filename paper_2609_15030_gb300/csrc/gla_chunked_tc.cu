@@ -172,6 +172,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     }
     if (warp == 0)
         tmem_alloc(sb + OFF_MISC, TMEM_COLS);
+    pdl_wait_and_release();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -268,9 +269,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         ph_tma ^= 1;
 
         if (L <= kShort) {
-            // ---- short segment: the per-token recurrence, with the recurrent kernel's
-            // exact operation order (two 64-row halves of each state column, each a
-            // sequential fma chain; o = half0 + half1), so both kernels agree bit for bit
+            // ---- short segment: the per-token recurrence with the recurrent kernel's exact
+            // operation order (fma chains over groups of 16 key rows, group partials summed
+            // left to right), so both kernels agree bit for bit
             for (int idx = tid; idx < L * D; idx += NT)
                 sG[idx] = expf(sG[idx]);
             __syncthreads();
@@ -278,17 +279,20 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             tmem_ld32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
             tmem_ld32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
             tmem_wait_ld();
-            float *part = reinterpret_cast<float *>(smem + OFF_A);   // [kShort][2][128]
+            float *part = reinterpret_cast<float *>(smem + OFF_QT);   // [kShort][8 groups][128]
             for (int i = 0; i < L; ++i) {
                 const float ve = bf16f(sV[i * D + e_own]);
-                float acc = 0.f;
 #pragma unroll
-                for (int r = 0; r < 64; ++r) {
-                    const int d = colhalf * 64 + r;
-                    S[r] = fmaf(sG[i * D + d], S[r], bf16f(sK[i * D + d]) * ve);
-                    acc = fmaf(bf16f(sQ[i * D + d]), S[r], acc);
+                for (int m = 0; m < 4; ++m) {
+                    float acc = 0.f;
+#pragma unroll
+                    for (int r = 16 * m; r < 16 * m + 16; ++r) {
+                        const int d = colhalf * 64 + r;
+                        S[r] = fmaf(sG[i * D + d], S[r], bf16f(sK[i * D + d]) * ve);
+                        acc = fmaf(bf16f(sQ[i * D + d]), S[r], acc);
+                    }
+                    part[(i * 8 + colhalf * 4 + m) * D + e_own] = acc;
                 }
-                part[(i * 2 + colhalf) * D + e_own] = acc;
             }
             tmem_st32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
             tmem_st32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
@@ -305,7 +309,11 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             float *ob = p.o + (((int64_t)b * p.max_tokens + tok) * p.n_heads + h) * D;
             for (int idx = tid; idx < L * D; idx += NT) {
                 const int i = idx >> 7, e = idx & (D - 1);
-                ob[(int64_t)i * tstride + e] = part[(i * 2) * D + e] + part[(i * 2 + 1) * D + e];
+                float sum = part[(i * 8) * D + e];
+#pragma unroll
+                for (int g = 1; g < 8; ++g)
+                    sum += part[(i * 8 + g) * D + e];
+                ob[(int64_t)i * tstride + e] = sum;
             }
             tc_fence_before();
             __syncthreads();
@@ -709,8 +717,7 @@ cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s)
     if (e != cudaSuccess)
         return e;
     const unsigned grid = (unsigned)p.batch * (unsigned)p.n_heads;
-    gla_chunked_tc_kernel<<<grid, NT, SMEM_BYTES, s>>>(p, maps);
-    return cudaGetLastError();
+    return launch_pdl(gla_chunked_tc_kernel, dim3(grid), dim3(NT), SMEM_BYTES, s, p, maps);
 }
 
 }  // namespace hs

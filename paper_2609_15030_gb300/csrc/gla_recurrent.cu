@@ -4,22 +4,23 @@
 // this is the form the library implements.)
 //
 // One CTA owns one (problem, head) and keeps its d x d float32 state in
-// registers for the whole call: thread (row group rg, column j) holds rows
-// [rg*R, rg*R+R) of column j.  Tokens are staged eight at a time in shared
-// memory; o_t is the fixed-order sum of the row groups' partial dot products.
-// Per token and element: g = expf(a), S = fmaf(g, S, k*v), partial =
-// fmaf(q, S, partial) in increasing row order; o = partial_0 + partial_1 + ...
-// The chunked tensor-core kernel runs short segments with exactly these
-// operations (d = 128), so the two kernels agree bit for bit on them.
-// The operation order per token depends only on the token's inputs and the
-// incoming state, so resuming from any checkpoint reproduces a full
-// recomputation bit for bit.
+// registers for the whole call, as 16 x 4 blocks (16 key rows, 4 value
+// columns) per thread, read and written as 16-byte vectors.  Tokens are
+// staged eight at a time in shared memory.
+//
+// Per token the arithmetic is fixed: g = expf(a); every element becomes
+// fmaf(g_d, S[d][e], k_d * v_e); partial dot products over each group of 16
+// consecutive key rows run as one sequential fma chain in increasing row
+// order; o_e is the left-to-right sum of the d/16 group partials.  The chunked
+// tensor-core kernel computes short segments with exactly these operations
+// (d = 128), so the two kernels agree bit for bit on them.  The order depends
+// only on each token's inputs and the incoming state, so resuming from any
+// checkpoint reproduces a full recomputation bit for bit.
 #include "hs_internal.cuh"
 
 namespace hs {
 namespace {
 
-constexpr int kThreads = 256;
 constexpr int kTokBlock = 8;
 
 __device__ __forceinline__ float bf16_to_f32(uint16_t x)
@@ -27,13 +28,17 @@ __device__ __forceinline__ float bf16_to_f32(uint16_t x)
     return __uint_as_float(((uint32_t)x) << 16);
 }
 
+// CTA = (problem, head).  Thread (cg, rg) holds the 16 x 4 block of the state
+// with rows [16*rg, 16*rg+16) and columns [4*cg, 4*cg+4): a warp covers 16-byte
+// pieces of whole rows, so state loads and stores are fully coalesced vectors.
 template <int D>
-__global__ void __launch_bounds__(kThreads) gla_recurrent_kernel(const __grid_constant__ GlaParams p)
+__global__ void __launch_bounds__((D / 4) * (D / 16)) gla_recurrent_kernel(const __grid_constant__ GlaParams p)
 {
-    constexpr int NG = kThreads / D;  // row groups
-    constexpr int R = D / NG;         // rows per thread
-    __shared__ float sq[kTokBlock][D], sk[kTokBlock][D], sg[kTokBlock][D], sv[kTokBlock][D];
-    __shared__ float spart[kTokBlock][NG][D];
+    constexpr int NCG = D / 4;        // column groups of 4
+    constexpr int NRG = D / 16;       // row groups of 16
+    constexpr int NTH = NCG * NRG;
+    __shared__ __align__(16) float sq[kTokBlock][D], sk[kTokBlock][D], sg[kTokBlock][D], sv[kTokBlock][D];
+    __shared__ __align__(16) float spart[kTokBlock][NRG][D];
 
     const int b = blockIdx.x / p.n_heads;
     const int h = blockIdx.x - b * p.n_heads;
@@ -41,20 +46,21 @@ __global__ void __launch_bounds__(kThreads) gla_recurrent_kernel(const __grid_co
     if (n <= 0)
         return;
     const int64_t pos0 = p.pos0[b];
+    pdl_wait_and_release();
     const int tid = threadIdx.x;
-    const int j = tid % D;
-    const int rg = tid / D;
+    const int cg = tid % NCG;
+    const int rg = tid / NCG;
     const int C = p.ckpt_interval;
 
     float *st = p.state + ((int64_t)b * p.n_heads + h) * D * D;
-    float S[R];
+    float4 S[16];   // S[r] = state row 16*rg + r, columns 4*cg .. 4*cg+3
 #pragma unroll
-    for (int r = 0; r < R; ++r)
-        S[r] = st[(int64_t)(rg * R + r) * D + j];
+    for (int r = 0; r < 16; ++r)
+        S[r] = *reinterpret_cast<const float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg);
 
     for (int t0 = 0; t0 < n; t0 += kTokBlock) {
         const int tb = min(kTokBlock, n - t0);
-        for (int idx = tid; idx < tb * D; idx += kThreads) {
+        for (int idx = tid; idx < tb * D; idx += NTH) {
             const int tt = idx / D, d = idx - (idx / D) * D;
             const int64_t row = ((int64_t)b * p.max_tokens + t0 + tt) * p.n_heads + h;
             sq[tt][d] = bf16_to_f32(p.q[row * D + d]);
@@ -64,15 +70,22 @@ __global__ void __launch_bounds__(kThreads) gla_recurrent_kernel(const __grid_co
         }
         __syncthreads();
         for (int tt = 0; tt < tb; ++tt) {
-            const float vj = sv[tt][j];
-            float acc = 0.f;
+            const float4 v4 = *reinterpret_cast<const float4 *>(&sv[tt][4 * cg]);
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-            for (int r = 0; r < R; ++r) {
-                const int i = rg * R + r;
-                S[r] = fmaf(sg[tt][i], S[r], sk[tt][i] * vj);
-                acc = fmaf(sq[tt][i], S[r], acc);
+            for (int r = 0; r < 16; ++r) {
+                const int i = 16 * rg + r;
+                const float g = sg[tt][i], kk = sk[tt][i], qq = sq[tt][i];
+                S[r].x = fmaf(g, S[r].x, kk * v4.x);
+                S[r].y = fmaf(g, S[r].y, kk * v4.y);
+                S[r].z = fmaf(g, S[r].z, kk * v4.z);
+                S[r].w = fmaf(g, S[r].w, kk * v4.w);
+                acc.x = fmaf(qq, S[r].x, acc.x);
+                acc.y = fmaf(qq, S[r].y, acc.y);
+                acc.z = fmaf(qq, S[r].z, acc.z);
+                acc.w = fmaf(qq, S[r].w, acc.w);
             }
-            spart[tt][rg][j] = acc;
+            *reinterpret_cast<float4 *>(&spart[tt][rg][4 * cg]) = acc;
             if (C > 0 && p.ckpt_slots != nullptr) {
                 const int64_t end = pos0 + t0 + tt + 1;
                 if (end % C == 0) {
@@ -87,27 +100,27 @@ __global__ void __launch_bounds__(kThreads) gla_recurrent_kernel(const __grid_co
                     } else {
                         slot += (int64_t)h * D * D;
 #pragma unroll
-                        for (int r = 0; r < R; ++r)
-                            slot[(int64_t)(rg * R + r) * D + j] = S[r];
+                        for (int r = 0; r < 16; ++r)
+                            *reinterpret_cast<float4 *>(slot + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
                     }
                 }
             }
         }
         __syncthreads();
-        for (int idx = tid; idx < tb * D; idx += kThreads) {
+        for (int idx = tid; idx < tb * D; idx += NTH) {
             const int tt = idx / D, e = idx - (idx / D) * D;
-            float s = spart[tt][0][e];
+            float sum = spart[tt][0][e];
 #pragma unroll
-            for (int g = 1; g < NG; ++g)
-                s += spart[tt][g][e];
+            for (int g = 1; g < NRG; ++g)
+                sum += spart[tt][g][e];
             const int64_t row = ((int64_t)b * p.max_tokens + t0 + tt) * p.n_heads + h;
-            p.o[row * D + e] = s;
+            p.o[row * D + e] = sum;
         }
         __syncthreads();
     }
 #pragma unroll
-    for (int r = 0; r < R; ++r)
-        st[(int64_t)(rg * R + r) * D + j] = S[r];
+    for (int r = 0; r < 16; ++r)
+        *reinterpret_cast<float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
 }
 
 }  // namespace
@@ -116,10 +129,8 @@ cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s)
 {
     const unsigned grid = (unsigned)p.batch * (unsigned)p.n_heads;
     if (d == 128)
-        gla_recurrent_kernel<128><<<grid, kThreads, 0, s>>>(p);
-    else
-        gla_recurrent_kernel<64><<<grid, kThreads, 0, s>>>(p);
-    return cudaGetLastError();
+        return launch_pdl(gla_recurrent_kernel<128>, dim3(grid), dim3(256), 0, s, p);
+    return launch_pdl(gla_recurrent_kernel<64>, dim3(grid), dim3(64), 0, s, p);
 }
 
 }  // namespace hs

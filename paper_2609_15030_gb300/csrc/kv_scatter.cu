@@ -33,6 +33,7 @@ kv_scatter_kernel(const void *const *staging, void *const *cache, int32_t n_laye
                   const int32_t *bt, int32_t n_pages, int64_t page_vecs, int64_t num_blocks,
                   int32_t *d_err)
 {
+    pdl_wait_and_release();
     const int64_t units = (int64_t)n_layers * n_pages;
     for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
         const int32_t l = (int32_t)(u / n_pages);
@@ -86,9 +87,8 @@ cudaError_t launch_kv_scatter(const void *const *staging, void *const *cache, in
     int64_t grid = (int64_t)sm_count * 8 * 4;
     if (grid > units)
         grid = units;
-    kv_scatter_kernel<<<(unsigned)grid, kThreads, 0, s>>>(staging, cache, n_layers, bt, n_pages,
-                                                          page_bytes / 16, num_blocks, d_err);
-    return cudaGetLastError();
+    return launch_pdl(kv_scatter_kernel, dim3((unsigned)grid), dim3(kThreads), 0, s, staging, cache,
+                      n_layers, bt, n_pages, (int64_t)(page_bytes / 16), num_blocks, d_err);
 }
 
 }  // namespace hs

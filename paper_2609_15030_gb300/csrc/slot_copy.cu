@@ -18,6 +18,7 @@ __global__ void __launch_bounds__(kThreads)
 slot_copy_kernel(const float *const *src, float *const *dst, int32_t n, int64_t floats_each,
                  int64_t pieces, int32_t *d_err)
 {
+    pdl_wait_and_release();
     const int64_t units = (int64_t)n * pieces;
     for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
         const int32_t i = (int32_t)(u / pieces);
@@ -71,8 +72,8 @@ cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t
     int64_t grid = (int64_t)sm_count * 8 * 2;
     if (grid > units)
         grid = units;
-    slot_copy_kernel<<<(unsigned)grid, kThreads, 0, s>>>(src, dst, n, floats_each, pieces, d_err);
-    return cudaGetLastError();
+    return launch_pdl(slot_copy_kernel, dim3((unsigned)grid), dim3(kThreads), 0, s, src, dst, n,
+                      floats_each, pieces, d_err);
 }
 
 }  // namespace hs
