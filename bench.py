@@ -20,6 +20,10 @@ timed on the host cores as a CPU baseline.
 
 ``--impl reference`` times the oracle itself (CPU) on a bounded sample of
 the same workload.
+
+``--case decode|prefill|kv`` runs one small piece of the workload a few
+times and prints its CUDA-event times (no JSON): the cases the committed ncu
+captures under profiles/ were taken on.
 """
 from __future__ import annotations
 
@@ -72,6 +76,23 @@ def gla_bytes(n_problems, n_heads, d, tokens_per_problem, ckpts_per_problem):
 
 def kv_bytes(n_layers, n_pages, page_bytes):
     return 2 * n_layers * n_pages * page_bytes
+
+
+KERNEL_OF = {"decode": "gla_recurrent_kernel<128>", "prefill": "gla_chunked_tc_kernel",
+             "restore": "kv_scatter_kernel+slot_copy_kernel"}
+
+
+def _traffic():
+    """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the
+    committed ncu captures listed in profiles/dram_traffic.txt ("kernel bytes" lines)."""
+    p = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    out = {}
+    if os.path.exists(p):
+        for line in open(p):
+            f = line.split()
+            if len(f) >= 2 and not line.startswith("#"):
+                out[f[0]] = int(float(f[1]))
+    return out
 
 
 # ---------------------------------------------------------------------------
@@ -508,16 +529,16 @@ def _cores():
         return os.cpu_count() or 1
 
 
-def cpu_baseline(n_samples=2):
+def cpu_baseline():
     cores = _cores()
-    samples = [OracleSample(r) for r in (0, N_REQ - 1)[:n_samples]]
+    samples = [OracleSample(r) for r in range(N_REQ)]
     t0 = time.perf_counter()
     toks = sum(s.run(cores) for s in samples)
     t = time.perf_counter() - t0
     return {"value": round(toks / t, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"{len(samples)} of the 9 requests (L=512 and L=4608, seed 0): align + page "
-                      "scatter + state copy + 256-token tail and 64 decode tokens of all 9 linear "
-                      f"layers x 16 heads, float64 token by token; {t:.1f} s wall"}
+            "sample": f"one step (the 9 requests of seed 0): align + page scatter + state copy + "
+                      "256-token tail and 64 decode tokens of all 9 linear layers x 16 heads, "
+                      f"float64 token by token; {t:.1f} s wall on {cores} threads"}
 
 
 def run_reference(args):
@@ -547,6 +568,68 @@ def run_reference(args):
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(val, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0}}))
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# small standalone cases for profiler captures
+# ---------------------------------------------------------------------------
+
+def run_case(name: str, iters: int = 5):
+    """decode: 64 single-token calls over 9 problems x 16 heads (d = 128);
+    prefill: one 256-token tail over 9 problems x 16 heads from pos0 = 4096 with
+    checkpoints every 256; kv: 12 layers x 256 pages x 64 KiB scattered into a
+    2,048-block cache.  Each repeated `iters` times on the current stream."""
+    import torch
+    import paper_2609_15030_gb300 as hs
+    from hs_inputs import torch_gen_linear, gen_block_table
+    from paper_2609_15030_gb300 import build
+    build.build()
+    dev = torch.device("cuda:0")
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    if name in ("decode", "prefill"):
+        B, nH, d = HYBRID12.n_lin, HYBRID12.n_heads, HYBRID12.d
+        T = DECODE_STEPS if name == "decode" else TAIL
+        q, k, v, a = torch_gen_linear(2, 0, B, T, nH, d, dev)
+        o = torch.empty((B, T, nH, d), device=dev)
+        st = torch.randn((B, nH, d, d), device=dev) * 0.5
+        slots = torch.empty((B, nH, d, d), device=dev)
+        ptrs = hs.ptr_array([slots[i] for i in range(B)], dev)
+        shape = hs.make_shape(B, nH, d, d, T)
+        tb, tbf = nH * d * 2, nH * d * 4
+        for it in range(iters):
+            ev[0].record()
+            if name == "decode":
+                for j in range(T):
+                    hs.hs_linattn_prefill_from_state(
+                        shape, q.data_ptr() + j * tb, k.data_ptr() + j * tb, v.data_ptr() + j * tb,
+                        a.data_ptr() + j * tbf, o.data_ptr() + j * tbf, st, [4096 + j] * B, [1] * B,
+                        0, None, None)
+            else:
+                hs.hs_linattn_prefill_from_state(shape, q, k, v, a, o, st, [4096] * B, [T] * B,
+                                                 HYBRID12.ckpt, ptrs, None)
+            ev[1].record()
+            torch.cuda.synchronize()
+            per = ev[0].elapsed_time(ev[1]) * 1e3 / (T if name == "decode" else 1)
+            print(f"{name} iter {it}: {per:.2f} us per call (host-launched)", flush=True)
+    elif name == "kv":
+        nL, n_pages, P, NB = 12, 256, KVSTRESS.page_bytes, 2048
+        st = torch.empty((nL, n_pages * P), dtype=torch.uint8, device=dev)
+        st.view(torch.int32).random_(generator=torch.Generator(device=dev).manual_seed(1))
+        cache = torch.empty((nL, NB * P), dtype=torch.uint8, device=dev)
+        sp = hs.ptr_array([st[l] for l in range(nL)], dev)
+        cp = hs.ptr_array([cache[l] for l in range(nL)], dev)
+        bt = torch.from_numpy(gen_block_table(9, 0, n_pages, NB)).to(dev)
+        for it in range(iters):
+            ev[0].record()
+            hs.hs_restore_kv_pages(sp, cp, nL, bt, n_pages, P, NB, None)
+            ev[1].record()
+            torch.cuda.synchronize()
+            t = ev[0].elapsed_time(ev[1]) * 1e-3
+            print(f"kv iter {it}: {t * 1e6:.1f} us, {kv_bytes(nL, n_pages, P) / t / 1e9:.0f} GB/s",
+                  flush=True)
+    else:
+        raise SystemExit(f"unknown case {name}")
     return 0
 
 
@@ -592,7 +675,11 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true",
                     help="skip TTFT arms, KV stress, e2e and CPU baseline")
+    ap.add_argument("--case", choices=["decode", "prefill", "kv"],
+                    help="run one small standalone case for a profiler capture")
     args = ap.parse_args()
+    if args.case:
+        return run_case(args.case)
     if args.impl == "reference":
         return run_reference(args)
     args.warmup = max(args.warmup, 3)
@@ -635,15 +722,19 @@ def main():
 
     peak, peak_kind = _peaks()
     groups = timer.summary()
-    gla = [groups[p] for p in ("prefill", "decode") if p in groups]
-    gla_nb = sum(g[0] for g in gla)
-    gla_ms = sum(g[1] for g in gla)
-    gla_n = sum(g[2] for g in gla)
-    achieved = gla_nb / (gla_ms * 1e-3) / 1e9
-    kernels = {k: {"launches": g[2], "ms": round(g[1], 3), "avg_us": round(g[1] * 1e3 / g[2], 2),
-                   "gbs": round(g[0] / (g[1] * 1e-3) / 1e9, 1),
-                   "share_of_step": round(g[1] * 1e-3 / t_local, 3)}
-               for k, g in groups.items()}
+    traffic = _traffic()
+
+    def roofline(phase):
+        nb, ms, n = groups[phase]
+        ach = nb / (ms * 1e-3) / 1e9
+        kern = KERNEL_OF[phase]
+        return {"bound": "hbm", "kernel": kern, "phase": phase, "achieved": round(ach, 1),
+                "peak": peak, "unit": "GB/s", "frac": round(ach / peak, 4), "peak_kind": peak_kind,
+                "traffic": traffic.get(kern), "bytes_per_launch": int(nb / n),
+                "avg_launch_us": round(ms * 1e3 / n, 3), "launches": n,
+                "share_of_step": round(ms * 1e-3 / t_local, 3)}
+
+    dominant = max(groups, key=lambda k: groups[k][1])
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t * 1e3 / args.steps, 3),
@@ -652,12 +743,8 @@ def main():
         "config": {"workload": WORKLOAD, "tokens_per_step": TOKENS_PER_STEP,
                    "l2": "inputs larger than L2: four seeds x nine requests rotate "
                          "(~2.7 GB of inputs), each step touches ~0.7 GB"},
-        "roofline": {"bound": "hbm", "kernel": "linear-attention prefill/decode (all launches)",
-                     "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                     "frac": round(achieved / peak, 4), "peak_kind": peak_kind,
-                     "traffic": None, "launches": gla_n,
-                     "avg_launch_us": round(gla_ms * 1e3 / max(gla_n, 1), 2)},
-        "kernels": kernels,
+        "roofline": roofline(dominant),
+        "roofline_by_phase": {k: roofline(k) for k in groups},
         "gpu_launches": launches,
         "clocks": clk,
     }
@@ -670,6 +757,7 @@ def main():
         torch.cuda.empty_cache()
         kv = kv_stress(dev)
         kv["frac"] = round(kv["gbs_aggregate"] / peak, 4)
+        kv["traffic"] = _traffic().get("kv_scatter_kernel@kvstress")
         out["kv_restore"] = kv
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
