@@ -54,39 +54,43 @@ using namespace ptx;
 
 constexpr int D = 128;    // d_k = d_v
 constexpr int CH = 64;    // chunk length (absolute grid)
-constexpr int NT = 256;   // threads per CTA
+constexpr int NW = 256;   // worker threads (warps 0..7): operands and epilogues
+constexpr int NT = NW + 32;  // + one warp whose lane 0 issues every MMA and TMA copy
+constexpr int kIssuer = NW;
 constexpr int kShort = 8; // segments of at most this many tokens run token by token
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kFastMinLog2 = -64.0f;      // factorised form if every 2^{Lam_last} >= 2^-64
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 
 // shared memory map (offsets from a 1024-byte aligned base).  Every tf32
-// operand is K-major (kind::tf32 takes no transposed shared-memory operand),
-// so the products that contract over tokens read V and K~ transposed.
+// shared-memory operand is K-major (kind::tf32 takes no transposed
+// shared-memory operand); V^T is the A operand of both token-contracting
+// products and lives in tensor memory.
 constexpr uint32_t OFF_QT = 0;          // Q~   [64 tok i][128 d]  tf32, swizzled   32 KiB
 constexpr uint32_t OFF_KT = 32768;      // K~   [64 tok j][128 d]                   32 KiB
-constexpr uint32_t OFF_KTT = 65536;     // K~^T [128 d][64 tok j] (K^^T on the exact path)  32 KiB
-constexpr uint32_t OFF_VT = 98304;      // V^T  [128 e][64 tok j]                   32 KiB
-constexpr uint32_t OFF_A = 131072;      // A    [64 i][64 j]                        16 KiB
-constexpr uint32_t OFF_SQ = 147456;     // staged q  bf16 [64][128]                16 KiB
-constexpr uint32_t OFF_SK = 163840;     // staged k                                 16 KiB
-constexpr uint32_t OFF_SV = 180224;     // staged v                                 16 KiB
-constexpr uint32_t OFF_SG = 196608;     // staged log-gates f32 [64][128]           32 KiB
-constexpr uint32_t OFF_GAM = 229376;    // 2^{Lam_last} per key dim                512 B
-constexpr uint32_t OFF_BAR = 229888;    // 4 mbarriers
-constexpr uint32_t OFF_MISC = 229920;   // TMEM base address, flags
-constexpr uint32_t SMEM_BYTES = 229936 + 1024;
+constexpr uint32_t OFF_B2 = 65536;      // [A ; K~^T] [64 i + 128 d][64 tok j]  (K^^T on the exact path)  48 KiB
+constexpr uint32_t OFF_SQ = 114688;     // staged q  bf16 [64][128]                16 KiB
+constexpr uint32_t OFF_SK = 131072;     // staged k                                 16 KiB
+constexpr uint32_t OFF_SV = 147456;     // staged v                                 16 KiB
+constexpr uint32_t OFF_SG = 163840;     // staged log-gates f32 [64][128]           32 KiB
+constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim                512 B
+constexpr uint32_t OFF_TOT = 197120;    // per-half log2-decay totals [2][128]      1 KiB
+constexpr uint32_t OFF_BAR = 198144;    // 4 mbarriers
+constexpr uint32_t OFF_MISC = 198176;   // TMEM base address, abort flag, exact-path flag
+constexpr uint32_t SMEM_BYTES = 198192 + 1024;
 constexpr uint32_t STAGE_BYTES = 3 * 16384 + 32768;
 constexpr uint32_t SLAB = 64 * 128;     // one 32-column slab of a 64-row operand
-constexpr uint32_t SLAB_T = 128 * 128;  // one 32-column slab of a 128-row operand
+constexpr uint32_t SLAB_B2 = 192 * 128; // one 32-column slab of the 192-row operand [A ; K~^T]
 
-constexpr uint32_t TMEM_COLS = 256;
-constexpr uint32_t TM_S = 0;            // S^T   128 lanes x 128 cols
-constexpr uint32_t TM_O = 128;          // D_O   128 lanes x 64 cols (lane e, col i)
+constexpr uint32_t TMEM_COLS = 512;
+constexpr uint32_t TM_O = 0;            // D_O   128 lanes x 64 cols (lane e, col i)
+constexpr uint32_t TM_S = 64;           // S^T   128 lanes x 128 cols; [D_O | S^T] is one N=192 accumulator
 constexpr uint32_t TM_A = 192;          // D_A   128 lanes x 64 cols (lanes 0..63 used)
+constexpr uint32_t TM_V = 256;          // V^T   128 lanes x 64 cols (lane e, col j)
 
 constexpr uint32_t IDESC_N64 = idesc_tf32(128, 64, 0, 0);    // M=128, N=64, K-major x K-major
 constexpr uint32_t IDESC_N128 = idesc_tf32(128, 128, 0, 0);  // M=128, N=128
+constexpr uint32_t IDESC_N192 = idesc_tf32(128, 192, 0, 0);  // M=128, N=192
 
 struct TmaMaps {
     CUtensorMap q, k, v, g;
@@ -101,10 +105,24 @@ __device__ __forceinline__ uint32_t sw_off(int row, int col)
                       ((col & 3) << 2));
 }
 
-// 16-byte chunk col4 (columns 4*col4 .. 4*col4+3) of row `row` of a 128-row operand
-__device__ __forceinline__ uint32_t sw_chunk_t(int row, int col4)
+// byte offset of element (i, j) of A = rows 0..63 of the 192-row operand [A ; K~^T]
+__device__ __forceinline__ uint32_t a_off(int i, int j)
 {
-    return (uint32_t)((col4 >> 3) * SLAB_T + row * 128 + (((col4 & 7) ^ (row & 7)) << 4));
+    return (uint32_t)((j >> 5) * SLAB_B2 + i * 128 + ((((j & 31) >> 2) ^ (i & 7)) << 4) + ((j & 3) << 2));
+}
+
+// 16-byte chunk col4 (tokens 4*col4 .. 4*col4+3) of row d of K~^T = rows 64..191 of [A ; K~^T]
+__device__ __forceinline__ uint32_t ktt_chunk(int d, int col4)
+{
+    return (uint32_t)((col4 >> 3) * SLAB_B2 + (64 + d) * 128 + (((col4 & 7) ^ (d & 7)) << 4));
+}
+
+__device__ __forceinline__ float warp_min(float v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
 }
 
 __device__ __forceinline__ float bf16f(uint16_t x)
@@ -195,12 +213,13 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tma_load_2d(sb + OFF_SG, &maps.g, x, y, bar_tma);
         tma_inflight = true;
     };
-    if (tid == 0)
+    if (tid == kIssuer)
         issue_tma(0);
 
     // incoming state -> TMEM, transposed: S^T[e][d] = state[d][e]
+    const bool worker = warp < 8;
     float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
-    {
+    if (worker) {
         float r[32];
 #pragma unroll
         for (int c0 = 0; c0 < 64; c0 += 32) {
@@ -213,23 +232,19 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tmem_wait_st();
     }
 
-    // operand-building map: thread owns key dims (dp, dp+1) of tokens [16*qr, 16*qr+16)
-    const int qr = lane >> 3;
-    const int dp = 2 * (warp * 8 + (lane & 7));
-    uint32_t nat[8];       // byte offset of (row 16*qr + r, col dp) in a 64-row operand
+    // operand-building map: thread owns key dim d = e_own for tokens [32*colhalf, +32);
+    // nat[r]: byte offset of (row 32*colhalf + r, col d) in a 64-row operand
+    const int d = e_own;
+    const int th = colhalf;
+    uint32_t nat[8];
     {
-        const uint32_t base = (uint32_t)((dp >> 5) * SLAB + (16 * qr) * 128 + ((dp & 3) << 2));
-        const int cd = (dp & 31) >> 2;
+        const uint32_t base = (uint32_t)((warp & 3) * SLAB + (32 * th) * 128 + ((lane & 3) << 2));
+        const int cd = lane >> 2;
 #pragma unroll
         for (int r = 0; r < 8; ++r)
             nat[r] = base + r * 128 + ((uint32_t)(cd ^ r) << 4);
     }
-    uint32_t tr0[4], tr1[4];   // 16-byte chunk (tokens 16*qr + 4g ..) of rows dp, dp+1 of a 128-row operand
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-        tr0[g] = sw_chunk_t(dp, 4 * qr + g);
-        tr1[g] = sw_chunk_t(dp + 1, 4 * qr + g);
-    }
+    float *sTot = reinterpret_cast<float *>(smem + OFF_TOT);
 
     tc_fence_before();
     __syncthreads();
@@ -255,13 +270,14 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
 
         // ---- 1. staged inputs
-        if (tid == 0) {
+        if (tid == kIssuer) {
             if (mbar_wait_bounded(bar_tma, ph_tma, kTimeoutNs))
                 tma_inflight = false;
             else
                 sMisc[1] = 1;
         }
         __syncthreads();
+        tc_fence_after();
         if (sMisc[1]) {
             aborted = true;
             break;
@@ -275,11 +291,12 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             for (int idx = tid; idx < L * D; idx += NT)
                 sG[idx] = expf(sG[idx]);
             __syncthreads();
+            float *part = reinterpret_cast<float *>(smem + OFF_QT);   // [kShort][8 groups][128]
             float S[64];
+            if (worker) {
             tmem_ld32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
             tmem_ld32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
             tmem_wait_ld();
-            float *part = reinterpret_cast<float *>(smem + OFF_QT);   // [kShort][8 groups][128]
             for (int i = 0; i < L; ++i) {
                 const float ve = bf16f(sV[i * D + e_own]);
 #pragma unroll
@@ -302,9 +319,10 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     slot[(int64_t)(colhalf * 64 + r) * D + e_own] = S[r];
             }
             tmem_wait_st();
+            }
             fence_proxy_async_smem();
             __syncthreads();
-            if (tid == 0 && has_next)
+            if (tid == kIssuer && has_next)
                 issue_tma(tok + L);
             float *ob = p.o + (((int64_t)b * p.max_tokens + tok) * p.n_heads + h) * D;
             for (int idx = tid; idx < L * D; idx += NT) {
@@ -341,120 +359,90 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             __syncthreads();
         }
 
-        // ---- 2. cumulative log2-gates: 16 tokens per thread, then a shuffle scan
-        //         over the four token quarters that hold the same key dims
-        float lam0[16], lam1[16];
-        float run0 = 0.f, run1 = 0.f;
+        // ---- 2. cumulative log2-gates: each thread scans its 32 tokens of key dim d;
+        //         the two token halves are joined through shared memory
+        float lam[32];
+        float run = 0.f;
+        if (worker) {
 #pragma unroll
-        for (int x = 0; x < 16; ++x) {
-            const float2 a2 = *reinterpret_cast<const float2 *>(sG + (16 * qr + x) * D + dp);
-            run0 = fmaf(a2.x, kLog2e, run0);
-            run1 = fmaf(a2.y, kLog2e, run1);
-            lam0[x] = run0;
-            lam1[x] = run1;
-        }
-        float s0 = run0, s1 = run1;
-        {
-            const float y0 = __shfl_up_sync(0xffffffffu, s0, 8);
-            const float y1 = __shfl_up_sync(0xffffffffu, s1, 8);
-            if (qr >= 1) {
-                s0 = s0 + y0;
-                s1 = s1 + y1;
+            for (int x = 0; x < 32; ++x) {
+                run = fmaf(sG[(32 * th + x) * D + d], kLog2e, run);
+                lam[x] = run;
             }
+            sTot[th * D + d] = run;
         }
-        {
-            const float y0 = __shfl_up_sync(0xffffffffu, s0, 16);
-            const float y1 = __shfl_up_sync(0xffffffffu, s1, 16);
-            if (qr >= 2) {
-                s0 = s0 + y0;
-                s1 = s1 + y1;
-            }
-        }
-        const float pre0 = __shfl_up_sync(0xffffffffu, s0, 8);   // tokens before this quarter
-        const float pre1 = __shfl_up_sync(0xffffffffu, s1, 8);
-        const float last0 = __shfl_sync(0xffffffffu, s0, (lane & 7) + 24);
-        const float last1 = __shfl_sync(0xffffffffu, s1, (lane & 7) + 24);
-        if (qr >= 1) {
+        if (tid == 0)
+            sMisc[2] = 0;   // exact-path flag of this segment
+        __syncthreads();
+        float last = 0.f;
+        if (worker) {
+            const float tot0 = sTot[d];
+            last = tot0 + sTot[D + d];   // Lam_last of key dim d
+            if (th) {
 #pragma unroll
-            for (int x = 0; x < 16; ++x) {
-                lam0[x] = pre0 + lam0[x];
-                lam1[x] = pre1 + lam1[x];
+                for (int x = 0; x < 32; ++x)
+                    lam[x] = tot0 + lam[x];
+            } else {
+                sGam[d] = ex2(last);
             }
+            // warp-shuffle min of the chunk's decay over this warp's key dims picks the path
+            const float wmin = warp_min(last);
+            if (lane == 0 && wmin < kFastMinLog2)
+                sMisc[2] = 1;
         }
-        if (qr == 0)
-            *reinterpret_cast<float2 *>(sGam + dp) = make_float2(ex2(last0), ex2(last1));
-        const bool slow = __syncthreads_or(last0 < kFastMinLog2 || last1 < kFastMinLog2) != 0;
 
-        // ---- operands (tf32, K-major, swizzled)
-        if (!slow) {
+        // ---- operands (tf32, K-major, swizzled), in two steps so the tensor core starts
+        //      early: Q~ (shared memory) and V^T (tensor memory) first, then S^T Q~^T runs
+        //      while K~ is built; Q~ K~^T then runs while K~^T is written
+        if (worker) {
+            float vtr[32];
 #pragma unroll
-            for (int g = 0; g < 4; ++g) {
-                float4 kt0, kt1, vt0, vt1;
-                float *k0 = &kt0.x, *k1 = &kt1.x, *v0 = &vt0.x, *v1 = &vt1.x;
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int x = 4 * g + u;
-                    const int i = 16 * qr + x;
-                    const uint32_t q2 = *reinterpret_cast<const uint32_t *>(sQ + i * D + dp);
-                    const uint32_t k2 = *reinterpret_cast<const uint32_t *>(sK + i * D + dp);
-                    const uint32_t v2 = *reinterpret_cast<const uint32_t *>(sV + i * D + dp);
-                    const uint32_t off = nat[x & 7] + (x >> 3) * 1024;
-                    *reinterpret_cast<float2 *>(smem + OFF_QT + off) =
-                        make_float2(rna_tf32(bf_lo(q2) * ex2(lam0[x])), rna_tf32(bf_hi(q2) * ex2(lam1[x])));
-                    const float ka = rna_tf32(bf_lo(k2) * ex2(-lam0[x]));
-                    const float kb = rna_tf32(bf_hi(k2) * ex2(-lam1[x]));
-                    *reinterpret_cast<float2 *>(smem + OFF_KT + off) = make_float2(ka, kb);
-                    k0[u] = ka;
-                    k1[u] = kb;
-                    v0[u] = bf_lo(v2);
-                    v1[u] = bf_hi(v2);
-                }
-                *reinterpret_cast<float4 *>(smem + OFF_KTT + tr0[g]) = kt0;
-                *reinterpret_cast<float4 *>(smem + OFF_KTT + tr1[g]) = kt1;
-                *reinterpret_cast<float4 *>(smem + OFF_VT + tr0[g]) = vt0;
-                *reinterpret_cast<float4 *>(smem + OFF_VT + tr1[g]) = vt1;
+            for (int x = 0; x < 32; ++x) {
+                const int i = 32 * th + x;
+                const float qv = bf16f(sQ[i * D + d]);
+                vtr[x] = bf16f(sV[i * D + d]);
+                *reinterpret_cast<float *>(smem + OFF_QT + nat[x & 7] + (x >> 3) * 1024) =
+                    rna_tf32(qv * ex2(lam[x]));
             }
-        } else {
-#pragma unroll 1
-            for (int g = 0; g < 4; ++g) {
-                float4 kt0, kt1, vt0, vt1;
-                float *k0 = &kt0.x, *k1 = &kt1.x, *v0 = &vt0.x, *v1 = &vt1.x;
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int x = 4 * g + u;
-                    const int i = 16 * qr + x;
-                    float la, lb;
-                    // dynamic index into lam (exact path only)
-#pragma unroll
-                    for (int z = 0; z < 16; ++z)
-                        if (z == x) {
-                            la = lam0[z];
-                            lb = lam1[z];
-                        }
-                    const uint32_t q2 = *reinterpret_cast<const uint32_t *>(sQ + i * D + dp);
-                    const uint32_t k2 = *reinterpret_cast<const uint32_t *>(sK + i * D + dp);
-                    const uint32_t v2 = *reinterpret_cast<const uint32_t *>(sV + i * D + dp);
-                    *reinterpret_cast<float2 *>(smem + OFF_QT + sw_off(i, dp)) =
-                        make_float2(rna_tf32(bf_lo(q2) * ex2(la)), rna_tf32(bf_hi(q2) * ex2(lb)));
-                    k0[u] = rna_tf32(bf_lo(k2) * ex2(last0 - la));   // K^ = k 2^{Lam_last - Lam}
-                    k1[u] = rna_tf32(bf_hi(k2) * ex2(last1 - lb));
-                    v0[u] = bf_lo(v2);
-                    v1[u] = bf_hi(v2);
-                    *reinterpret_cast<float2 *>(sG + i * D + dp) = make_float2(la, lb);
-                }
-                *reinterpret_cast<float4 *>(smem + OFF_KTT + sw_chunk_t(dp, 4 * qr + g)) = kt0;
-                *reinterpret_cast<float4 *>(smem + OFF_KTT + sw_chunk_t(dp + 1, 4 * qr + g)) = kt1;
-                *reinterpret_cast<float4 *>(smem + OFF_VT + sw_chunk_t(dp, 4 * qr + g)) = vt0;
-                *reinterpret_cast<float4 *>(smem + OFF_VT + sw_chunk_t(dp + 1, 4 * qr + g)) = vt1;
-            }
+            tmem_st32(tmem + lrow + TM_V + 32 * th, vtr);
+            tmem_wait_st();
         }
         fence_proxy_async_smem();
+        tc_fence_before();
         __syncthreads();
-
-        // ---- 3a. first MMA group
-        if (tid == 0) {
+        const bool slow = sMisc[2] != 0;
+        if (tid == kIssuer) {
+            // ---- 3a. S^T Q~^T into D_O (A operand read from tensor memory)
             tc_fence_after();
-            if (!slow) {
+#pragma unroll
+            for (int kk = 0; kk < D / 8; ++kk) {
+                const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
+                mma_tf32_ts(tmem + TM_O, tmem + TM_S + kk * 8,
+                            sdesc_sw128(sb + OFF_QT + koff, 16, 1024), IDESC_N64, kk > 0);
+            }
+        }
+        if (!slow) {
+            if (worker) {
+                // K~ token-major (operand of Q~ K~^T) and transposed (operand of the state update)
+#pragma unroll
+                for (int g = 0; g < 8; ++g) {
+                    float4 kt4;
+                    float *kv4 = &kt4.x;
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const int x = 4 * g + u;
+                        const int i = 32 * th + x;
+                        kv4[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(-lam[x]));
+                        *reinterpret_cast<float *>(smem + OFF_KT + nat[x & 7] + (x >> 3) * 1024) = kv4[u];
+                    }
+                    *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(d, 8 * th + g)) = kt4;
+                }
+            }
+            fence_proxy_async_smem();
+            __syncthreads();
+            if (tid == kIssuer) {
+                // ---- Q~ K~^T into D_A; the staging buffers are free for the next segment
+                tc_fence_after();
 #pragma unroll
                 for (int kk = 0; kk < D / 8; ++kk) {
                     const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
@@ -462,20 +450,12 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                                 sdesc_sw128(sb + OFF_KT + koff, 16, 1024), IDESC_N64, kk > 0);
                 }
                 tc_commit(bar_a);
+                if (has_next)
+                    issue_tma(tok + L);
             }
-#pragma unroll
-            for (int kk = 0; kk < D / 8; ++kk) {
-                const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
-                mma_tf32_ts(tmem + TM_O, tmem + TM_S + kk * 8,
-                            sdesc_sw128(sb + OFF_QT + koff, 16, 1024), IDESC_N64, kk > 0);
-            }
-            if (!slow && has_next)
-                issue_tma(tok + L);
-        }
 
-        // ---- 3b. the causally masked intra-chunk matrix A -> shared memory
-        if (!slow) {
-            if (tid == 0 && !mbar_wait_bounded(bar_a, ph_a, kTimeoutNs))
+            // ---- 3b. the causally masked intra-chunk matrix A -> shared memory
+            if (tid == kIssuer && !mbar_wait_bounded(bar_a, ph_a, kTimeoutNs))
                 sMisc[1] = 1;
             __syncthreads();
             if (sMisc[1]) {
@@ -484,7 +464,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             ph_a ^= 1;
             tc_fence_after();
-            if ((warp & 3) < 2) {
+            if (worker && (warp & 3) < 2) {
                 const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
                 const int jb = (warp >> 2) * 32;            // this warp's 32 key columns
                 float r[32];
@@ -497,12 +477,32 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
                         wv[u] = (jb + 4 * c + u <= i) ? rna_tf32(r[4 * c + u]) : 0.f;
-                    const uint32_t o = (jb >> 5) * SLAB + i * 128 + ((uint32_t)(c ^ (i & 7)) << 4);
-                    *reinterpret_cast<float4 *>(smem + OFF_A + o) = w;
+                    const uint32_t o = (jb >> 5) * SLAB_B2 + i * 128 + ((uint32_t)(c ^ (i & 7)) << 4);
+                    *reinterpret_cast<float4 *>(smem + OFF_B2 + o) = w;
                 }
             }
         } else {
-            // exact elementwise path: A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}, j <= i < L
+            // ---- exact path: K^ = k 2^{Lam_last - Lam} (transposed) and the cumulative
+            //      log2-gates in place, then A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}
+            if (worker)
+#pragma unroll
+            for (int g = 0; g < 8; ++g) {
+                float4 w;
+                float *wv = &w.x;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int x = 4 * g + u;
+                    const int i = 32 * th + x;
+                    wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam[x]));
+                }
+                *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(d, 8 * th + g)) = w;
+            }
+            __syncthreads();   // every thread has read its log-gates before they are overwritten
+            if (worker)
+#pragma unroll
+            for (int x = 0; x < 32; ++x)
+                sG[(32 * th + x) * D + d] = lam[x];
+            __syncthreads();
             for (int idx = tid; idx < CH * CH; idx += NT) {
                 const int i = idx >> 6, j = idx & 63;
                 float acc = 0.f;
@@ -511,31 +511,25 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                         acc = fmaf(bf16f(sQ[i * D + dd]) * bf16f(sK[j * D + dd]),
                                    ex2(sG[i * D + dd] - sG[j * D + dd]), acc);
                 }
-                *reinterpret_cast<float *>(smem + OFF_A + sw_off(i, j)) = rna_tf32(acc);
+                *reinterpret_cast<float *>(smem + OFF_B2 + a_off(i, j)) = rna_tf32(acc);
             }
         }
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
 
-        // ---- 3c. second MMA group
-        if (tid == 0) {
+        // ---- 3c. second MMA group: [D_O | S^T] += V^T [A ; K~^T]^T on the factorised path
+        //          (one N=192 product), D_O += V^T A^T alone on the exact path; the A
+        //          operand V^T is read from tensor memory
+        if (tid == kIssuer) {
             tc_fence_after();
             if (slow && has_next)
                 issue_tma(tok + L);
 #pragma unroll
             for (int kk = 0; kk < CH / 8; ++kk) {
-                const uint64_t va = sdesc_sw128(sb + OFF_VT + (kk >> 2) * SLAB_T + (kk & 3) * 32, 16, 1024);
-                const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
-                mma_tf32_ss(tmem + TM_O, va, sdesc_sw128(sb + OFF_A + koff, 16, 1024), IDESC_N64, 1);
-            }
-            if (!slow) {
-#pragma unroll
-                for (int kk = 0; kk < CH / 8; ++kk) {
-                    const uint32_t koff = (kk >> 2) * SLAB_T + (kk & 3) * 32;
-                    mma_tf32_ss(tmem + TM_S, sdesc_sw128(sb + OFF_VT + koff, 16, 1024),
-                                sdesc_sw128(sb + OFF_KTT + koff, 16, 1024), IDESC_N128, 1);
-                }
+                const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32;
+                mma_tf32_ts(tmem + TM_O, tmem + TM_V + kk * 8, sdesc_sw128(sb + OFF_B2 + koff, 16, 1024),
+                            slow ? IDESC_N64 : IDESC_N192, 1);
             }
             tc_commit(bar_o);
             if (!mbar_wait_bounded(bar_o, ph_o, kTimeoutNs))
@@ -550,7 +544,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tc_fence_after();
 
         // ---- 4a. outputs: lane e holds o[i][e] for 32 rows i
-        {
+        if (worker) {
             float r[32];
             const int ib = colhalf * 32;
             tmem_ld32(tmem + lrow + TM_O + ib, r);
@@ -569,6 +563,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
 
         // ---- 4b. state decay (after the update on the factorised path, before it on the exact path)
+        if (worker)
 #pragma unroll
         for (int c0 = 0; c0 < 64; c0 += 32) {
             const int d0 = colhalf * 64 + c0;
@@ -594,13 +589,13 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (slow) {
             tc_fence_before();
             __syncthreads();
-            if (tid == 0) {
+            if (tid == kIssuer) {
                 tc_fence_after();
 #pragma unroll
                 for (int kk = 0; kk < CH / 8; ++kk) {
-                    const uint32_t koff = (kk >> 2) * SLAB_T + (kk & 3) * 32;
-                    mma_tf32_ss(tmem + TM_S, sdesc_sw128(sb + OFF_VT + koff, 16, 1024),
-                                sdesc_sw128(sb + OFF_KTT + koff, 16, 1024), IDESC_N128, 1);
+                    const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32 + 64 * 128;
+                    mma_tf32_ts(tmem + TM_S, tmem + TM_V + kk * 8,
+                                sdesc_sw128(sb + OFF_B2 + koff, 16, 1024), IDESC_N128, 1);
                 }
                 tc_commit(bar_s);
                 if (!mbar_wait_bounded(bar_s, ph_s, kTimeoutNs))
@@ -613,7 +608,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             ph_s ^= 1;
             tc_fence_after();
-            if (slot != nullptr) {
+            if (worker && slot != nullptr) {
 #pragma unroll
                 for (int c0 = 0; c0 < 64; c0 += 32) {
                     const int d0 = colhalf * 64 + c0;
@@ -626,14 +621,16 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 }
             }
         }
+        // no barrier here: the next segment's first barrier orders these TMEM stores
+        // before its MMAs, and nothing below reads what this epilogue wrote
         tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
         pos = seg_end;
         tok += L;
     }
+    __syncthreads();
+    tc_fence_after();
 
-    if (!aborted) {
+    if (!aborted && worker) {
         // final state back to global memory, row = key dim
         float r[32];
 #pragma unroll
@@ -645,7 +642,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             for (int x = 0; x < 32; ++x)
                 st_g[(int64_t)(d0 + x) * D + e_own] = r[x];
         }
-    } else if (tid == 0) {
+    } else if (aborted && tid == kIssuer) {
         report(p.d_err, HS_DEVERR_TIMEOUT);
         // let this CTA's own copies and MMAs drain (bounded) before its memory goes away
         if (tma_inflight)
