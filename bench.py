@@ -23,7 +23,8 @@ the same workload.
 
 ``--case decode|prefill|kv`` runs one small piece of the workload a few
 times and prints its CUDA-event times (no JSON): the cases the committed ncu
-captures under profiles/ were taken on.
+captures under profiles/ were taken on.  ``--case long`` prints resumed vs
+recomputed TTFT for the long-context stack (L = 16k/32k/64k, batch 4).
 """
 from __future__ import annotations
 
@@ -628,8 +629,89 @@ def run_case(name: str, iters: int = 5):
             t = ev[0].elapsed_time(ev[1]) * 1e-3
             print(f"kv iter {it}: {t * 1e6:.1f} us, {kv_bytes(nL, n_pages, P) / t / 1e9:.0f} GB/s",
                   flush=True)
+    elif name == "long":
+        return run_long(dev)
     else:
         raise SystemExit(f"unknown case {name}")
+    return 0
+
+
+def run_long(dev):
+    """Long-context hybrid stack: 24 layers (18 linear: 32 heads, d = 128, C = 512;
+    6 full: 8 KV heads, head_dim 128, page 32), batch 4, L in {16k, 32k, 64k},
+    complete hit (c = L - 512) and partial hit L - 37 (same c).  Resumed TTFT =
+    align + KV restore of [0,c) for 6 layers + state restore of 18 layers + the
+    512-token tail prefill of every linear layer; recomputation = prefill of
+    [0,L) from the zero state emitting every checkpoint + the KV write of L
+    tokens.  One q/k/v/gate set per request is shared by the 18 linear layers
+    (18 distinct sets at L = 64k would need ~190 GB), so each layer is one call."""
+    import torch
+    import paper_2609_15030_gb300 as hs
+    from hs_inputs import LONG24, LONG_LENGTHS, torch_gen_linear, torch_fill_bf16_normal
+    S = LONG24
+    B, nH, d, nL, nF, P, C = S.batch, S.n_heads, S.d, S.n_lin, S.n_full, S.page, S.ckpt
+    Lmax = max(LONG_LENGTHS)
+    q, k, v, a = torch_gen_linear(7, 0, B, Lmax, nH, d, dev)
+    o = torch.empty((B, Lmax, nH, d), device=dev)
+    states = torch.zeros((nL, B, nH, d, d), device=dev)
+    nck = Lmax // C
+    slots = torch.empty((B * nck, nH, d, d), device=dev)
+    pb = S.page_bytes
+    n_pages_max = Lmax // P
+    NB = B * n_pages_max + 64
+    cache = torch.empty((nF, NB * pb), dtype=torch.uint8, device=dev)
+    staging = torch.empty((B, nF, n_pages_max * pb), dtype=torch.uint8, device=dev)
+    torch_fill_bf16_normal(staging, 3)
+    cache_ptrs = hs.ptr_array([cache[l] for l in range(nF)], dev)
+    stg_ptrs = [hs.ptr_array([staging[b, l] for l in range(nF)], dev) for b in range(B)]
+    perm = torch.randperm(NB, device=dev).to(torch.int32)
+    bts = [perm[b * n_pages_max:(b + 1) * n_pages_max].contiguous() for b in range(B)]
+    ck_src = torch.randn((nL, B, nH, d, d), device=dev) * 0.5
+    src_ptrs = hs.ptr_array([ck_src[l] for l in range(nL)], dev)
+    dst_ptrs = hs.ptr_array([states[l] for l in range(nL)], dev)
+    ev = lambda: torch.cuda.Event(enable_timing=True)
+    print(json.dumps({"case": "long", "workload": "long-24L (18 linear 32h d128 C512 + 6 full 8kv hd128 P32), batch 4"}))
+    for Lc in LONG_LENGTHS:
+        # complete hit; cached prefix L-37 of an L-token prompt; an (L-37)-token prompt
+        # fully cached (ragged tail inside the last chunk)
+        for L, hit in ((Lc, Lc), (Lc, Lc - 37), (Lc - 37, Lc - 37)):
+            c, n_pages, tail = hs.hs_align_prefix(L, hit, list(range(C, L + 1, C)), P)
+            # resumed
+            shape_t = hs.make_shape(B, nH, d, d, Lmax)
+            slot_ptrs = hs.ptr_array([slots[b] for b in range(B)], dev) if L % C == 0 else None
+            tok = c * nH * d
+            def resume():
+                for b in range(B):
+                    hs.hs_restore_kv_pages(stg_ptrs[b], cache_ptrs, nF, bts[b], n_pages, pb, NB)
+                hs.hs_restore_state(src_ptrs, dst_ptrs, nL, B * nH * d * d)
+                for l in range(nL):
+                    hs.hs_linattn_prefill_from_state(
+                        shape_t, q.data_ptr() + 2 * tok, k.data_ptr() + 2 * tok, v.data_ptr() + 2 * tok,
+                        a.data_ptr() + 4 * tok, o.data_ptr() + 4 * tok, states[l], [c] * B, [tail] * B, C,
+                        slot_ptrs)
+            per = L // C
+            ckp = hs.ptr_array([slots[b * nck + m] for b in range(B) for m in range(per)], dev)
+            if hs.hs_linattn_num_checkpoints([c] * B, [tail] * B, C) != (B if L % C == 0 else 0):
+                raise SystemExit("unexpected checkpoint count")
+            def recompute():
+                for l in range(nL):
+                    states[l].zero_()
+                    hs.hs_linattn_prefill_from_state(shape_t, q, k, v, a, o, states[l], [0] * B, [L] * B, C, ckp)
+                for b in range(B):
+                    hs.hs_restore_kv_pages(stg_ptrs[b], cache_ptrs, nF, bts[b], L // P, pb, NB)
+            res = {}
+            for nm, fn in (("resume", resume), ("recompute", recompute)):
+                fn()
+                torch.cuda.synchronize(dev)
+                e0, e1 = ev(), ev()
+                e0.record()
+                fn()
+                e1.record()
+                torch.cuda.synchronize(dev)
+                res[nm] = e0.elapsed_time(e1)
+            print(json.dumps({"L": L, "hit": hit, "c": c, "tail": tail, "ttft_resume_ms": round(res["resume"], 3),
+                              "ttft_recompute_ms": round(res["recompute"], 3),
+                              "ratio": round(res["recompute"] / res["resume"], 1)}), flush=True)
     return 0
 
 
@@ -675,7 +757,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true",
                     help="skip TTFT arms, KV stress, e2e and CPU baseline")
-    ap.add_argument("--case", choices=["decode", "prefill", "kv"],
+    ap.add_argument("--case", choices=["decode", "prefill", "kv", "long"],
                     help="run one small standalone case for a profiler capture")
     args = ap.parse_args()
     if args.case:

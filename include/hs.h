@@ -199,6 +199,10 @@ typedef struct hs_linattn_shape {
  *   log_g      device float [batch][max_tokens][n_heads][d_k]
  *   o          device float [batch][max_tokens][n_heads][d_v]; rows t >= n_tokens[b]
  *              are not written
+ *              max_tokens is the token stride between problems; only rows
+ *              t < n_tokens[b] of each problem are read or written, so views that start
+ *              mid-sequence (pointer offset by whole tokens) are valid as long as those
+ *              rows exist.
  *   state      device float [batch][n_heads][d_k][d_v], row index = key dimension
  *   pos0       host int64 [batch], >= 0
  *   n_tokens   host int32 [batch], 0 <= n_tokens[b] <= max_tokens

@@ -96,14 +96,6 @@ struct TmaMaps {
     CUtensorMap q, k, v, g;
 };
 
-// Byte offset of element (row, col) of a row-major f32 operand stored as
-// 32-column slabs (128-byte rows) in the 128-byte swizzled K-major canonical
-// layout: 16-byte chunk c of row r sits at chunk position c ^ (r % 8).
-__device__ __forceinline__ uint32_t sw_off(int row, int col)
-{
-    return (uint32_t)((col >> 5) * SLAB + row * 128 + ((((col & 31) >> 2) ^ (row & 7)) << 4) +
-                      ((col & 3) << 2));
-}
 
 // byte offset of element (i, j) of A = rows 0..63 of the 192-row operand [A ; K~^T]
 __device__ __forceinline__ uint32_t a_off(int i, int j)
@@ -130,15 +122,7 @@ __device__ __forceinline__ float bf16f(uint16_t x)
     return __uint_as_float(((uint32_t)x) << 16);
 }
 
-__device__ __forceinline__ float bf_lo(uint32_t w)
-{
-    return __uint_as_float(w << 16);
-}
 
-__device__ __forceinline__ float bf_hi(uint32_t w)
-{
-    return __uint_as_float(w & 0xFFFF0000u);
-}
 
 // 2^x, one MUFU op (relative error ~2^-22; inputs here lie in [-2^7, 2^7])
 __device__ __forceinline__ float ex2(float x)
@@ -701,7 +685,11 @@ cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s)
         return cudaErrorNotSupported;
     TmaMaps maps;
     const uint64_t inner = (uint64_t)p.n_heads * D;
-    const uint64_t rows = (uint64_t)p.batch * (uint64_t)p.max_tokens;
+    // rows up to the last problem's last token: copies never read beyond the tokens the
+    // caller passed (boxes reaching further are zero-filled), so q/k/v/log_g may be
+    // offset views whose batch stride runs past the end of the allocation
+    const uint64_t rows = (uint64_t)(p.batch - 1) * (uint64_t)p.max_tokens +
+                          (uint64_t)p.n_tokens[p.batch - 1];
     if (rows == 0)
         return cudaSuccess;
     if (!encode_rows(&maps.q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.q, inner, rows, 2) ||

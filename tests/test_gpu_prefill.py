@@ -296,3 +296,32 @@ def test_table4_suffix_lengths_auto_resume_bitwise(suffix):
     o_f, S_f, ck_f, = _resume_equals_recompute(inp, N, c, C, dev, hs.HS_LINATTN_AUTO)
     ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], C_=C)
     _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], f"suffix={suffix}")
+
+
+@pytest.mark.parametrize("kernel", KERNELS)
+def test_offset_views_read_only_the_given_tokens(kernel):
+    """Views that start mid-sequence (pointer offset by c tokens, batch stride kept)
+    read and write only rows t < n_tokens: the last problem's rows end exactly at the
+    end of the allocation, and results equal those of a contiguous copy, bitwise."""
+    dev = device()
+    B, T, nH, d, c = 3, 320, 2, 128, 192
+    inp = gen_linear(15, 0, B, T, nH, d, d)
+    S0 = gen_state(15, 0, B, nH, d, d)
+    sub = type(inp)(*(np.ascontiguousarray(x[:, c:]) for x in (inp.q, inp.k, inp.v, inp.a)))
+    o_ref, S_ref, _ = run_prefill(sub, [c] * B, [T - c] * B, S0, 0, dev, kernel, want_ckpts=False)
+    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    o = torch.full((B, T, nH, d), 7.0, device=dev)
+    state = to_dev(S0, dev)
+    off = c * nH * d
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_linattn_prefill_from_state(hs.make_shape(B, nH, d, d, T, kernel),
+                                     q.data_ptr() + 2 * off, k.data_ptr() + 2 * off,
+                                     v.data_ptr() + 2 * off, a.data_ptr() + 4 * off,
+                                     o.data_ptr() + 4 * off, state, [c] * B, [T - c] * B, 0, None,
+                                     err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    got = o.cpu().numpy()
+    assert np.array_equal(got[:, c:].view(np.uint32), o_ref[:, :T - c].view(np.uint32))
+    assert (got[:, :c] == 7.0).all()
+    assert np.array_equal(state.cpu().numpy().view(np.uint32), S_ref.view(np.uint32))
