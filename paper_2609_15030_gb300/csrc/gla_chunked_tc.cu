@@ -73,20 +73,25 @@ constexpr uint32_t OFF_SQ = 114688;     // staged q  bf16 [64][128]             
 constexpr uint32_t OFF_SK = 131072;     // staged k                                 16 KiB
 constexpr uint32_t OFF_SV = 147456;     // staged v                                 16 KiB
 constexpr uint32_t OFF_SG = 163840;     // staged log-gates f32 [64][128]           32 KiB
-constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim                512 B
-constexpr uint32_t OFF_TOT = 197120;    // per-half log2-decay totals [2][128]      1 KiB
-constexpr uint32_t OFF_BAR = 198144;    // 4 mbarriers
-constexpr uint32_t OFF_MISC = 198176;   // TMEM base address, abort flag, exact-path flag
-constexpr uint32_t SMEM_BYTES = 198192 + 1024;
+constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim, one buffer per chunk parity   1 KiB
+constexpr uint32_t OFF_TOT = 197632;    // per-half log2-decay totals [2][128]      1 KiB
+constexpr uint32_t OFF_BAR = 198656;    // 4 mbarriers
+constexpr uint32_t OFF_MISC = 198688;   // TMEM base address, abort flag, exact-path flags (per parity)
+constexpr uint32_t SMEM_BYTES = 198720 + 1024;
 constexpr uint32_t STAGE_BYTES = 3 * 16384 + 32768;
 constexpr uint32_t SLAB = 64 * 128;     // one 32-column slab of a 64-row operand
 constexpr uint32_t SLAB_B2 = 192 * 128; // one 32-column slab of the 192-row operand [A ; K~^T]
 
+// tensor memory: the output accumulator D_O alternates between two buffers by chunk
+// parity, placed on either side of S^T so that [D_O0 | S^T] and [S^T | D_O1] are each one
+// N=192 accumulator; V^T alternates likewise.  Even chunks order the 192-row operand as
+// [A ; K~^T], odd chunks as [K~^T ; A].
 constexpr uint32_t TMEM_COLS = 512;
-constexpr uint32_t TM_O = 0;            // D_O   128 lanes x 64 cols (lane e, col i)
-constexpr uint32_t TM_S = 64;           // S^T   128 lanes x 128 cols; [D_O | S^T] is one N=192 accumulator
-constexpr uint32_t TM_A = 192;          // D_A   128 lanes x 64 cols (lanes 0..63 used)
-constexpr uint32_t TM_V = 256;          // V^T   128 lanes x 64 cols (lane e, col j)
+constexpr uint32_t TM_O0 = 0;           // D_O of even chunks (lane e, col i), 64 cols
+constexpr uint32_t TM_S = 64;           // S^T  128 lanes x 128 cols
+constexpr uint32_t TM_O1 = 192;         // D_O of odd chunks
+constexpr uint32_t TM_A = 256;          // D_A  128 lanes x 64 cols (lanes 0..63 used)
+constexpr uint32_t TM_V = 320;          // V^T  2 x 64 cols (lane e, col j)
 
 constexpr uint32_t IDESC_N64 = idesc_tf32(128, 64, 0, 0);    // M=128, N=64, K-major x K-major
 constexpr uint32_t IDESC_N128 = idesc_tf32(128, 128, 0, 0);  // M=128, N=128
@@ -97,16 +102,17 @@ struct TmaMaps {
 };
 
 
-// byte offset of element (i, j) of A = rows 0..63 of the 192-row operand [A ; K~^T]
-__device__ __forceinline__ uint32_t a_off(int i, int j)
+// byte offset of element (i, j) of A, stored from row rowA of the 192-row operand
+__device__ __forceinline__ uint32_t a_off(int rowA, int i, int j)
 {
-    return (uint32_t)((j >> 5) * SLAB_B2 + i * 128 + ((((j & 31) >> 2) ^ (i & 7)) << 4) + ((j & 3) << 2));
+    return (uint32_t)((j >> 5) * SLAB_B2 + (rowA + i) * 128 + ((((j & 31) >> 2) ^ (i & 7)) << 4) +
+                      ((j & 3) << 2));
 }
 
-// 16-byte chunk col4 (tokens 4*col4 .. 4*col4+3) of row d of K~^T = rows 64..191 of [A ; K~^T]
-__device__ __forceinline__ uint32_t ktt_chunk(int d, int col4)
+// 16-byte chunk col4 (tokens 4*col4 .. 4*col4+3) of row d of K~^T, stored from row rowK
+__device__ __forceinline__ uint32_t ktt_chunk(int rowK, int d, int col4)
 {
-    return (uint32_t)((col4 >> 3) * SLAB_B2 + (64 + d) * 128 + (((col4 & 7) ^ (d & 7)) << 4));
+    return (uint32_t)((col4 >> 3) * SLAB_B2 + (rowK + d) * 128 + (((col4 & 7) ^ (d & 7)) << 4));
 }
 
 __device__ __forceinline__ float warp_min(float v)
@@ -149,7 +155,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     const uint16_t *sK = reinterpret_cast<const uint16_t *>(smem + OFF_SK);
     const uint16_t *sV = reinterpret_cast<const uint16_t *>(smem + OFF_SV);
     float *sG = reinterpret_cast<float *>(smem + OFF_SG);
-    float *sGam = reinterpret_cast<float *>(smem + OFF_GAM);
+    float *sTot = reinterpret_cast<float *>(smem + OFF_TOT);
     volatile uint32_t *sMisc = reinterpret_cast<volatile uint32_t *>(smem + OFF_MISC);
     const uint32_t bar_tma = sb + OFF_BAR, bar_a = sb + OFF_BAR + 8, bar_o = sb + OFF_BAR + 16,
                    bar_s = sb + OFF_BAR + 24;
@@ -163,6 +169,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     const int64_t pos0 = p.pos0[b];
     const int64_t end = pos0 + n;
     const int64_t tstride = (int64_t)p.n_heads * D;   // elements between consecutive tokens
+    const int C = p.ckpt_interval;
 
     if (tid == 0) {
         mbar_init(bar_tma, 1);
@@ -179,13 +186,26 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sMisc[0];
+    const bool worker = warp < 8;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
     const int colhalf = warp >> 2;
     const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
+    // operand-building map: worker owns key dim d = e_own for tokens [32*th, 32*th+32)
+    const int d = e_own;
+    const int th = colhalf;
+    uint32_t nat[8];       // byte offset of (row 32*th + r, col d) in a 64-row operand
+    {
+        const uint32_t base = (uint32_t)((warp & 3) * SLAB + (32 * th) * 128 + ((lane & 3) << 2));
+        const int cd = lane >> 2;
+#pragma unroll
+        for (int r = 0; r < 8; ++r)
+            nat[r] = base + r * 128 + ((uint32_t)(cd ^ r) << 4);
+    }
 
-    // thread-0 bookkeeping of work in flight (for the abort path)
+    // issuer bookkeeping (lane 0 of warp 8) of work in flight, for the abort path
     bool tma_inflight = false;
     uint32_t ph_tma = 0, ph_a = 0, ph_o = 0, ph_s = 0;
+    bool aborted = false;
 
     auto issue_tma = [&](int64_t tok_local) {
         const int32_t y = (int32_t)((int64_t)b * p.max_tokens + tok_local);
@@ -197,11 +217,42 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tma_load_2d(sb + OFF_SG, &maps.g, x, y, bar_tma);
         tma_inflight = true;
     };
+    // the issuer waits on an mbarrier, then everyone meets; false if a wait ran out
+    auto wait_all = [&](uint32_t bar, uint32_t &ph) -> bool {
+        if (tid == kIssuer && !mbar_wait_bounded(bar, ph, kTimeoutNs))
+            sMisc[1] = 1;
+        __syncthreads();
+        tc_fence_after();
+        ph ^= 1;
+        if (sMisc[1]) {
+            aborted = true;
+            return false;
+        }
+        return true;
+    };
+    auto wait_tma = [&]() -> bool {
+        const bool ok = wait_all(bar_tma, ph_tma);
+        if (tid == kIssuer)
+            tma_inflight = false;
+        return ok;
+    };
+    auto seg_len = [&](int64_t at) -> int { return (int)(min(end, (at / CH + 1) * CH) - at); };
+    auto ckpt_slot = [&](int64_t seg_end) -> float * {
+        if (!(C > 0 && seg_end % C == 0 && p.ckpt_slots != nullptr))
+            return nullptr;
+        float *slot = p.ckpt_slots[p.ck_base[b] + (seg_end / C - pos0 / C - 1)];
+        if (slot == nullptr || (reinterpret_cast<uintptr_t>(slot) & 15u) != 0) {
+            if (tid == 0)
+                report(p.d_err, slot == nullptr ? HS_DEVERR_NULL : HS_DEVERR_MISALIGNED);
+            return nullptr;
+        }
+        return slot + (int64_t)h * D * D;
+    };
+
     if (tid == kIssuer)
         issue_tma(0);
 
     // incoming state -> TMEM, transposed: S^T[e][d] = state[d][e]
-    const bool worker = warp < 8;
     float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
     if (worker) {
         float r[32];
@@ -215,69 +266,21 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
         tmem_wait_st();
     }
-
-    // operand-building map: thread owns key dim d = e_own for tokens [32*colhalf, +32);
-    // nat[r]: byte offset of (row 32*colhalf + r, col d) in a 64-row operand
-    const int d = e_own;
-    const int th = colhalf;
-    uint32_t nat[8];
-    {
-        const uint32_t base = (uint32_t)((warp & 3) * SLAB + (32 * th) * 128 + ((lane & 3) << 2));
-        const int cd = lane >> 2;
-#pragma unroll
-        for (int r = 0; r < 8; ++r)
-            nat[r] = base + r * 128 + ((uint32_t)(cd ^ r) << 4);
-    }
-    float *sTot = reinterpret_cast<float *>(smem + OFF_TOT);
-
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
 
-    const int C = p.ckpt_interval;
-    int64_t pos = pos0, tok = 0;
-    bool aborted = false;
-    while (pos < end) {
-        const int64_t seg_end = min(end, (pos / CH + 1) * CH);
-        const int L = (int)(seg_end - pos);
-        const bool has_next = seg_end < end;
-        float *slot = nullptr;     // checkpoint slot of this segment's end, if any
-        if (C > 0 && seg_end % C == 0 && p.ckpt_slots != nullptr) {
-            slot = p.ckpt_slots[p.ck_base[b] + (seg_end / C - pos0 / C - 1)];
-            if (slot == nullptr || (reinterpret_cast<uintptr_t>(slot) & 15u) != 0) {
-                if (tid == 0)
-                    report(p.d_err, slot == nullptr ? HS_DEVERR_NULL : HS_DEVERR_MISALIGNED);
-                slot = nullptr;
-            } else {
-                slot += (int64_t)h * D * D;
-            }
-        }
-
-        // ---- 1. staged inputs
-        if (tid == kIssuer) {
-            if (mbar_wait_bounded(bar_tma, ph_tma, kTimeoutNs))
-                tma_inflight = false;
-            else
-                sMisc[1] = 1;
-        }
+    // ---- a short segment (<= kShort tokens, staged inputs already waited for): the
+    // per-token recurrence with the recurrent kernel's exact operation order (fma chains
+    // over groups of 16 key rows, group partials summed left to right)
+    auto short_segment = [&](int64_t tok_s, int L, int64_t seg_end) {
+        for (int idx = tid; idx < L * D; idx += NT)
+            sG[idx] = expf(sG[idx]);
         __syncthreads();
-        tc_fence_after();
-        if (sMisc[1]) {
-            aborted = true;
-            break;
-        }
-        ph_tma ^= 1;
-
-        if (L <= kShort) {
-            // ---- short segment: the per-token recurrence with the recurrent kernel's exact
-            // operation order (fma chains over groups of 16 key rows, group partials summed
-            // left to right), so both kernels agree bit for bit
-            for (int idx = tid; idx < L * D; idx += NT)
-                sG[idx] = expf(sG[idx]);
-            __syncthreads();
-            float *part = reinterpret_cast<float *>(smem + OFF_QT);   // [kShort][8 groups][128]
+        float *part = reinterpret_cast<float *>(smem + OFF_QT);   // [kShort][8 groups][128]
+        float *slot = ckpt_slot(seg_end);
+        if (worker) {
             float S[64];
-            if (worker) {
             tmem_ld32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
             tmem_ld32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
             tmem_wait_ld();
@@ -288,9 +291,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     float acc = 0.f;
 #pragma unroll
                     for (int r = 16 * m; r < 16 * m + 16; ++r) {
-                        const int d = colhalf * 64 + r;
-                        S[r] = fmaf(sG[i * D + d], S[r], bf16f(sK[i * D + d]) * ve);
-                        acc = fmaf(bf16f(sQ[i * D + d]), S[r], acc);
+                        const int dd = colhalf * 64 + r;
+                        S[r] = fmaf(sG[i * D + dd], S[r], bf16f(sK[i * D + dd]) * ve);
+                        acc = fmaf(bf16f(sQ[i * D + dd]), S[r], acc);
                     }
                     part[(i * 8 + colhalf * 4 + m) * D + e_own] = acc;
                 }
@@ -303,30 +306,33 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     slot[(int64_t)(colhalf * 64 + r) * D + e_own] = S[r];
             }
             tmem_wait_st();
-            }
-            fence_proxy_async_smem();
-            __syncthreads();
-            if (tid == kIssuer && has_next)
-                issue_tma(tok + L);
-            float *ob = p.o + (((int64_t)b * p.max_tokens + tok) * p.n_heads + h) * D;
-            for (int idx = tid; idx < L * D; idx += NT) {
-                const int i = idx >> 7, e = idx & (D - 1);
-                float sum = part[(i * 8) * D + e];
-#pragma unroll
-                for (int g = 1; g < 8; ++g)
-                    sum += part[(i * 8 + g) * D + e];
-                ob[(int64_t)i * tstride + e] = sum;
-            }
-            tc_fence_before();
-            __syncthreads();
-            tc_fence_after();
-            pos = seg_end;
-            tok += L;
-            continue;
         }
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (tid == kIssuer && seg_end < end)
+            issue_tma(tok_s + L);
+        float *ob = p.o + (((int64_t)b * p.max_tokens + tok_s) * p.n_heads + h) * D;
+        for (int idx = tid; idx < L * D; idx += NT) {
+            const int i = idx >> 7, e = idx & (D - 1);
+            float sum = part[(i * 8) * D + e];
+#pragma unroll
+            for (int g = 1; g < 8; ++g)
+                sum += part[(i * 8 + g) * D + e];
+            ob[(int64_t)i * tstride + e] = sum;
+        }
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+    };
 
+    // ---- prep of a long segment (staged inputs already waited for): zero the staged rows
+    // past the segment, cumulative log2-gates (per-thread scan of 32 tokens, halves joined
+    // through shared memory, path vote by a warp-shuffle min), Q~ into shared memory and
+    // V^T into tensor memory buffer `par`.  Leaves lam[] in registers.
+    float lam[32];
+    float last = 0.f;
+    auto prep = [&](int L, int par) {
         if (L < CH) {
-            // zero the staged rows past the segment: every operand row >= L becomes 0
             for (int idx = tid; idx < (CH - L) * 80; idx += NT) {
                 const int row = L + idx / 80, c = idx % 80;
                 uint4 *dst;
@@ -342,10 +348,6 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             __syncthreads();
         }
-
-        // ---- 2. cumulative log2-gates: each thread scans its 32 tokens of key dim d;
-        //         the two token halves are joined through shared memory
-        float lam[32];
         float run = 0.f;
         if (worker) {
 #pragma unroll
@@ -356,9 +358,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             sTot[th * D + d] = run;
         }
         if (tid == 0)
-            sMisc[2] = 0;   // exact-path flag of this segment
+            sMisc[2 + par] = 0;   // exact-path flag of this segment
         __syncthreads();
-        float last = 0.f;
         if (worker) {
             const float tot0 = sTot[d];
             last = tot0 + sTot[D + d];   // Lam_last of key dim d
@@ -367,18 +368,11 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 for (int x = 0; x < 32; ++x)
                     lam[x] = tot0 + lam[x];
             } else {
-                sGam[d] = ex2(last);
+                reinterpret_cast<float *>(smem + OFF_GAM)[par * D + d] = ex2(last);
             }
-            // warp-shuffle min of the chunk's decay over this warp's key dims picks the path
             const float wmin = warp_min(last);
             if (lane == 0 && wmin < kFastMinLog2)
-                sMisc[2] = 1;
-        }
-
-        // ---- operands (tf32, K-major, swizzled), in two steps so the tensor core starts
-        //      early: Q~ (shared memory) and V^T (tensor memory) first, then S^T Q~^T runs
-        //      while K~ is built; Q~ K~^T then runs while K~^T is written
-        if (worker) {
+                sMisc[2 + par] = 1;
             float vtr[32];
 #pragma unroll
             for (int x = 0; x < 32; ++x) {
@@ -388,67 +382,178 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 *reinterpret_cast<float *>(smem + OFF_QT + nat[x & 7] + (x >> 3) * 1024) =
                     rna_tf32(qv * ex2(lam[x]));
             }
-            tmem_st32(tmem + lrow + TM_V + 32 * th, vtr);
+            tmem_st32(tmem + lrow + TM_V + 64 * par + 32 * th, vtr);
             tmem_wait_st();
         }
         fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        const bool slow = sMisc[2] != 0;
-        if (tid == kIssuer) {
-            // ---- 3a. S^T Q~^T into D_O (A operand read from tensor memory)
-            tc_fence_after();
+    };
+
+    // ---- output epilogue of a processed segment: D_O buffer `par` -> o (lane e, 32 rows)
+    auto out_epilogue = [&](int64_t tok_s, int L, int par) {
+        if (!worker)
+            return;
+        float r[32];
+        const int ib = colhalf * 32;
+        tmem_ld32(tmem + lrow + (par ? TM_O1 : TM_O0) + ib, r);
+        tmem_wait_ld();
+        float *op = p.o + (((int64_t)b * p.max_tokens + tok_s + ib) * p.n_heads + h) * D + e_own;
+        if (L == CH) {
 #pragma unroll
-            for (int kk = 0; kk < D / 8; ++kk) {
-                const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
-                mma_tf32_ts(tmem + TM_O, tmem + TM_S + kk * 8,
-                            sdesc_sw128(sb + OFF_QT + koff, 16, 1024), IDESC_N64, kk > 0);
+            for (int x = 0; x < 32; ++x)
+                __stcs(op + (int64_t)x * tstride, r[x]);
+        } else {
+#pragma unroll
+            for (int x = 0; x < 32; ++x)
+                if (ib + x < L)
+                    __stcs(op + (int64_t)x * tstride, r[x]);
+        }
+    };
+
+    // ---- state decay by 2^{Lam_last} (buffer `par`), checkpoint from the same registers
+    auto decay_state = [&](int par, float *slot) {
+        if (!worker)
+            return;
+        const float *gam = reinterpret_cast<const float *>(smem + OFF_GAM) + par * D;
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 32) {
+            const int d0 = colhalf * 64 + c0;
+            float r[32];
+            tmem_ld32(tmem + lrow + TM_S + d0, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+                const float4 g4 = *reinterpret_cast<const float4 *>(gam + d0 + 4 * c);
+                r[4 * c] *= g4.x;
+                r[4 * c + 1] *= g4.y;
+                r[4 * c + 2] *= g4.z;
+                r[4 * c + 3] *= g4.w;
+            }
+            tmem_st32(tmem + lrow + TM_S + d0, r);
+            if (slot != nullptr) {
+#pragma unroll
+                for (int x = 0; x < 32; ++x)
+                    slot[(int64_t)(d0 + x) * D + e_own] = r[x];
             }
         }
-        if (!slow) {
-            if (worker) {
-                // K~ token-major (operand of Q~ K~^T) and transposed (operand of the state update)
-#pragma unroll
-                for (int g = 0; g < 8; ++g) {
-                    float4 kt4;
-                    float *kv4 = &kt4.x;
-#pragma unroll
-                    for (int u = 0; u < 4; ++u) {
-                        const int x = 4 * g + u;
-                        const int i = 32 * th + x;
-                        kv4[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(-lam[x]));
-                        *reinterpret_cast<float *>(smem + OFF_KT + nat[x & 7] + (x >> 3) * 1024) = kv4[u];
-                    }
-                    *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(d, 8 * th + g)) = kt4;
-                }
-            }
-            fence_proxy_async_smem();
+        tmem_wait_st();
+    };
+
+    int64_t pos = pos0, tok = 0;
+    // leading short segment
+    if (seg_len(pos) <= kShort) {
+        if (!wait_tma())
+            goto finish;
+        short_segment(tok, seg_len(pos), pos + seg_len(pos));
+        tok += seg_len(pos);
+        pos += seg_len(pos);
+    }
+
+    // ---- pipelined long segments
+    if (pos < end && seg_len(pos) > kShort) {
+        if (!wait_tma())
+            goto finish;
+        prep(seg_len(pos), 0);
+        int par = 0;
+        bool prev_valid = false;
+        int64_t tok_prev = 0;
+        int L_prev = 0;
+        while (true) {
+            const int L = seg_len(pos);
+            const int64_t seg_end = pos + L;
+            const bool has_next = seg_end < end;
+            const int L_next = has_next ? seg_len(seg_end) : 0;
+            const bool next_long = has_next && L_next > kShort;
+            const uint32_t rowA = par ? 128u : 0u, rowK = par ? 0u : 64u;
+            const uint32_t tm_o = par ? TM_O1 : TM_O0;
+
+            // Q~ / V^T of this segment and the previous decay are complete
+            tc_fence_before();
             __syncthreads();
+            const bool slow = sMisc[2 + par] != 0;
             if (tid == kIssuer) {
-                // ---- Q~ K~^T into D_A; the staging buffers are free for the next segment
+                // S^T Q~^T into D_O[par] (A operand read from tensor memory)
                 tc_fence_after();
 #pragma unroll
                 for (int kk = 0; kk < D / 8; ++kk) {
                     const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
-                    mma_tf32_ss(tmem + TM_A, sdesc_sw128(sb + OFF_QT + koff, 16, 1024),
-                                sdesc_sw128(sb + OFF_KT + koff, 16, 1024), IDESC_N64, kk > 0);
+                    mma_tf32_ts(tmem + tm_o, tmem + TM_S + kk * 8,
+                                sdesc_sw128(sb + OFF_QT + koff, 16, 1024), IDESC_N64, kk > 0);
                 }
-                tc_commit(bar_a);
-                if (has_next)
-                    issue_tma(tok + L);
             }
-
-            // ---- 3b. the causally masked intra-chunk matrix A -> shared memory
-            if (tid == kIssuer && !mbar_wait_bounded(bar_a, ph_a, kTimeoutNs))
-                sMisc[1] = 1;
+            if (worker) {
+                if (!slow) {
+                    // K~ token-major (operand of Q~ K~^T) and transposed (state update)
+#pragma unroll
+                    for (int g = 0; g < 8; ++g) {
+                        float4 kt4;
+                        float *kv4 = &kt4.x;
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const int x = 4 * g + u;
+                            const int i = 32 * th + x;
+                            kv4[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(-lam[x]));
+                            *reinterpret_cast<float *>(smem + OFF_KT + nat[x & 7] + (x >> 3) * 1024) = kv4[u];
+                        }
+                        *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(rowK, d, 8 * th + g)) = kt4;
+                    }
+                } else {
+                    // exact path: K^ = k 2^{Lam_last - Lam} (transposed), cumulative log2-gates
+                    // token-major in the (unused) K~ buffer
+#pragma unroll
+                    for (int g = 0; g < 8; ++g) {
+                        float4 w;
+                        float *wv = &w.x;
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const int x = 4 * g + u;
+                            const int i = 32 * th + x;
+                            wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam[x]));
+                            reinterpret_cast<float *>(smem + OFF_KT)[i * D + d] = lam[x];
+                        }
+                        *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(rowK, d, 8 * th + g)) = w;
+                    }
+                }
+            }
+            fence_proxy_async_smem();
             __syncthreads();
-            if (sMisc[1]) {
-                aborted = true;
-                break;
+            if (slow) {
+                // A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}, j <= i < L, elementwise
+                const float *lg = reinterpret_cast<const float *>(smem + OFF_KT);
+                for (int idx = tid; idx < CH * CH; idx += NT) {
+                    const int i = idx >> 6, j = idx & 63;
+                    float acc = 0.f;
+                    if (j <= i && i < L) {
+                        for (int dd = 0; dd < D; ++dd)
+                            acc = fmaf(bf16f(sQ[i * D + dd]) * bf16f(sK[j * D + dd]),
+                                       ex2(lg[i * D + dd] - lg[j * D + dd]), acc);
+                    }
+                    *reinterpret_cast<float *>(smem + OFF_B2 + a_off(rowA, i, j)) = rna_tf32(acc);
+                }
+                fence_proxy_async_smem();
+                __syncthreads();
             }
-            ph_a ^= 1;
-            tc_fence_after();
-            if (worker && (warp & 3) < 2) {
+            if (tid == kIssuer) {
+                tc_fence_after();
+                if (!slow) {
+                    // Q~ K~^T into D_A
+#pragma unroll
+                    for (int kk = 0; kk < D / 8; ++kk) {
+                        const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
+                        mma_tf32_ss(tmem + TM_A, sdesc_sw128(sb + OFF_QT + koff, 16, 1024),
+                                    sdesc_sw128(sb + OFF_KT + koff, 16, 1024), IDESC_N64, kk > 0);
+                    }
+                }
+                tc_commit(bar_a);     // covers S^T Q~^T too: Q~ is free once it arrives
+                if (has_next)
+                    issue_tma(tok + L);   // the staged inputs have been consumed
+            }
+            // output of the previous segment while the tensor core works
+            if (prev_valid)
+                out_epilogue(tok_prev, L_prev, par ^ 1);
+            if (!wait_all(bar_a, ph_a))
+                break;
+            if (!slow && worker && (warp & 3) < 2) {
+                // the causally masked intra-chunk matrix A -> rows rowA.. of [A ; K~^T]
                 const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
                 const int jb = (warp >> 2) * 32;            // this warp's 32 key columns
                 float r[32];
@@ -461,172 +566,111 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
                         wv[u] = (jb + 4 * c + u <= i) ? rna_tf32(r[4 * c + u]) : 0.f;
-                    const uint32_t o = (jb >> 5) * SLAB_B2 + i * 128 + ((uint32_t)(c ^ (i & 7)) << 4);
+                    const uint32_t o = (jb >> 5) * SLAB_B2 + (rowA + i) * 128 + ((uint32_t)(c ^ (i & 7)) << 4);
                     *reinterpret_cast<float4 *>(smem + OFF_B2 + o) = w;
                 }
             }
-        } else {
-            // ---- exact path: K^ = k 2^{Lam_last - Lam} (transposed) and the cumulative
-            //      log2-gates in place, then A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}
-            if (worker)
-#pragma unroll
-            for (int g = 0; g < 8; ++g) {
-                float4 w;
-                float *wv = &w.x;
-#pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int x = 4 * g + u;
-                    const int i = 32 * th + x;
-                    wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam[x]));
-                }
-                *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(d, 8 * th + g)) = w;
-            }
-            __syncthreads();   // every thread has read its log-gates before they are overwritten
-            if (worker)
-#pragma unroll
-            for (int x = 0; x < 32; ++x)
-                sG[(32 * th + x) * D + d] = lam[x];
-            __syncthreads();
-            for (int idx = tid; idx < CH * CH; idx += NT) {
-                const int i = idx >> 6, j = idx & 63;
-                float acc = 0.f;
-                if (j <= i && i < L) {
-                    for (int dd = 0; dd < D; ++dd)
-                        acc = fmaf(bf16f(sQ[i * D + dd]) * bf16f(sK[j * D + dd]),
-                                   ex2(sG[i * D + dd] - sG[j * D + dd]), acc);
-                }
-                *reinterpret_cast<float *>(smem + OFF_B2 + a_off(i, j)) = rna_tf32(acc);
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-
-        // ---- 3c. second MMA group: [D_O | S^T] += V^T [A ; K~^T]^T on the factorised path
-        //          (one N=192 product), D_O += V^T A^T alone on the exact path; the A
-        //          operand V^T is read from tensor memory
-        if (tid == kIssuer) {
-            tc_fence_after();
-            if (slow && has_next)
-                issue_tma(tok + L);
-#pragma unroll
-            for (int kk = 0; kk < CH / 8; ++kk) {
-                const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32;
-                mma_tf32_ts(tmem + TM_O, tmem + TM_V + kk * 8, sdesc_sw128(sb + OFF_B2 + koff, 16, 1024),
-                            slow ? IDESC_N64 : IDESC_N192, 1);
-            }
-            tc_commit(bar_o);
-            if (!mbar_wait_bounded(bar_o, ph_o, kTimeoutNs))
-                sMisc[1] = 1;
-        }
-        __syncthreads();
-        if (sMisc[1]) {
-            aborted = true;
-            break;
-        }
-        ph_o ^= 1;
-        tc_fence_after();
-
-        // ---- 4a. outputs: lane e holds o[i][e] for 32 rows i
-        if (worker) {
-            float r[32];
-            const int ib = colhalf * 32;
-            tmem_ld32(tmem + lrow + TM_O + ib, r);
-            tmem_wait_ld();
-            float *op = p.o + (((int64_t)b * p.max_tokens + tok + ib) * p.n_heads + h) * D + e_own;
-            if (L == CH) {
-#pragma unroll
-                for (int x = 0; x < 32; ++x)
-                    __stcs(op + (int64_t)x * tstride, r[x]);
-            } else {
-#pragma unroll
-                for (int x = 0; x < 32; ++x)
-                    if (ib + x < L)
-                        __stcs(op + (int64_t)x * tstride, r[x]);
-            }
-        }
-
-        // ---- 4b. state decay (after the update on the factorised path, before it on the exact path)
-        if (worker)
-#pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 32) {
-            const int d0 = colhalf * 64 + c0;
-            float r[32];
-            tmem_ld32(tmem + lrow + TM_S + d0, r);
-            tmem_wait_ld();
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                const float4 g4 = *reinterpret_cast<const float4 *>(sGam + d0 + 4 * c);
-                r[4 * c] *= g4.x;
-                r[4 * c + 1] *= g4.y;
-                r[4 * c + 2] *= g4.z;
-                r[4 * c + 3] *= g4.w;
-            }
-            tmem_st32(tmem + lrow + TM_S + d0, r);
-            if (!slow && slot != nullptr) {
-#pragma unroll
-                for (int x = 0; x < 32; ++x)
-                    slot[(int64_t)(d0 + x) * D + e_own] = r[x];
-            }
-        }
-        tmem_wait_st();
-        if (slow) {
+            fence_proxy_async_smem();
             tc_fence_before();
             __syncthreads();
             if (tid == kIssuer) {
+                // [D_O | S^T] += V^T [A ; K~^T]^T as one N=192 product (V^T from tensor
+                // memory); on the exact path only D_O += V^T A^T here
                 tc_fence_after();
+                const uint32_t vt = tmem + TM_V + 64 * par;
 #pragma unroll
                 for (int kk = 0; kk < CH / 8; ++kk) {
-                    const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32 + 64 * 128;
-                    mma_tf32_ts(tmem + TM_S, tmem + TM_V + kk * 8,
-                                sdesc_sw128(sb + OFF_B2 + koff, 16, 1024), IDESC_N128, 1);
+                    const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32;
+                    if (!slow)
+                        mma_tf32_ts(tmem + (par ? TM_S : TM_O0), vt + kk * 8,
+                                    sdesc_sw128(sb + OFF_B2 + koff, 16, 1024), IDESC_N192, 1);
+                    else
+                        mma_tf32_ts(tmem + tm_o, vt + kk * 8,
+                                    sdesc_sw128(sb + OFF_B2 + koff + rowA * 128, 16, 1024), IDESC_N64, 1);
                 }
-                tc_commit(bar_s);
-                if (!mbar_wait_bounded(bar_s, ph_s, kTimeoutNs))
-                    sMisc[1] = 1;
+                tc_commit(bar_o);
             }
-            __syncthreads();
-            if (sMisc[1]) {
-                aborted = true;
+            // next segment's inputs while the tensor core runs the second product
+            if (next_long) {
+                if (!wait_tma())
+                    break;
+                prep(L_next, par ^ 1);
+            }
+            if (!wait_all(bar_o, ph_o))
                 break;
-            }
-            ph_s ^= 1;
-            tc_fence_after();
-            if (worker && slot != nullptr) {
+            float *slot = ckpt_slot(seg_end);
+            decay_state(par, slow ? nullptr : slot);
+            if (slow) {
+                tc_fence_before();
+                __syncthreads();
+                if (tid == kIssuer) {
+                    tc_fence_after();
+                    const uint32_t vt = tmem + TM_V + 64 * par;
 #pragma unroll
-                for (int c0 = 0; c0 < 64; c0 += 32) {
-                    const int d0 = colhalf * 64 + c0;
-                    float r[32];
-                    tmem_ld32(tmem + lrow + TM_S + d0, r);
-                    tmem_wait_ld();
+                    for (int kk = 0; kk < CH / 8; ++kk) {
+                        const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32 + rowK * 128;
+                        mma_tf32_ts(tmem + TM_S, vt + kk * 8, sdesc_sw128(sb + OFF_B2 + koff, 16, 1024),
+                                    IDESC_N128, 1);
+                    }
+                    tc_commit(bar_s);
+                }
+                if (!wait_all(bar_s, ph_s))
+                    break;
+                if (worker && slot != nullptr) {
 #pragma unroll
-                    for (int x = 0; x < 32; ++x)
-                        slot[(int64_t)(d0 + x) * D + e_own] = r[x];
+                    for (int c0 = 0; c0 < 64; c0 += 32) {
+                        const int d0 = colhalf * 64 + c0;
+                        float r[32];
+                        tmem_ld32(tmem + lrow + TM_S + d0, r);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int x = 0; x < 32; ++x)
+                            slot[(int64_t)(d0 + x) * D + e_own] = r[x];
+                    }
                 }
             }
+            prev_valid = true;
+            tok_prev = tok;
+            L_prev = L;
+            pos = seg_end;
+            tok += L;
+            par ^= 1;
+            if (!next_long)
+                break;
         }
-        // no barrier here: the next segment's first barrier orders these TMEM stores
-        // before its MMAs, and nothing below reads what this epilogue wrote
+        if (aborted)
+            goto finish;
+        // output of the last pipelined segment
+        out_epilogue(tok_prev, L_prev, par ^ 1);
         tc_fence_before();
-        pos = seg_end;
-        tok += L;
+        __syncthreads();
+        tc_fence_after();
     }
-    __syncthreads();
-    tc_fence_after();
 
-    if (!aborted && worker) {
-        // final state back to global memory, row = key dim
-        float r[32];
+    // trailing short segment (its inputs were requested by the previous segment)
+    if (pos < end) {
+        if (!wait_tma())
+            goto finish;
+        short_segment(tok, seg_len(pos), pos + seg_len(pos));
+        pos += seg_len(pos);
+    }
+
+finish:
+    if (!aborted) {
+        if (worker) {
+            // final state back to global memory, row = key dim
+            float r[32];
 #pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 32) {
-            const int d0 = colhalf * 64 + c0;
-            tmem_ld32(tmem + lrow + TM_S + d0, r);
-            tmem_wait_ld();
+            for (int c0 = 0; c0 < 64; c0 += 32) {
+                const int d0 = colhalf * 64 + c0;
+                tmem_ld32(tmem + lrow + TM_S + d0, r);
+                tmem_wait_ld();
 #pragma unroll
-            for (int x = 0; x < 32; ++x)
-                st_g[(int64_t)(d0 + x) * D + e_own] = r[x];
+                for (int x = 0; x < 32; ++x)
+                    st_g[(int64_t)(d0 + x) * D + e_own] = r[x];
+            }
         }
-    } else if (aborted && tid == kIssuer) {
+    } else if (tid == kIssuer) {
         report(p.d_err, HS_DEVERR_TIMEOUT);
         // let this CTA's own copies and MMAs drain (bounded) before its memory goes away
         if (tma_inflight)
@@ -641,6 +685,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tmem_dealloc(tmem, TMEM_COLS);
     }
 }
+
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 {
