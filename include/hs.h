@@ -108,8 +108,9 @@ hs_status hs_align_prefix(int64_t N, int64_t hit_len, const int64_t *avail_ckpts
  *     cache_layers[l] + block_table[j]*page_bytes  <-  staging_layers[l] + j*page_bytes
  * (page_bytes bytes).  Bytes of the cache outside the listed blocks are not
  * written.
- *   staging_layers  device array of n_layers device pointers, each to
- *                   n_pages*page_bytes bytes laid out page after page
+ *   staging_layers  device array of n_layers pointers, each to n_pages*page_bytes
+ *                   bytes laid out page after page; device memory, or pinned host memory
+ *                   the device can address (the pages are then read over the host link)
  *   cache_layers    device array of n_layers device pointers, each to
  *                   num_blocks*page_bytes bytes (one layer's paged cache)
  *   block_table     device, n_pages int32 block ids; ids must be distinct (two equal

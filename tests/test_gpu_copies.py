@@ -154,3 +154,25 @@ def test_state_copy_null_slot_reports():
     torch.cuda.synchronize()
     assert err.item() == hs.HS_DEVERR_NULL
     assert torch.equal(b, a)
+
+
+def test_scatter_from_pinned_host_staging():
+    """Staging pages in pinned host memory (device-accessible): the scatter reads them
+    directly over the host link, as the paper's CPU cache tier is read (Section 5.5)."""
+    dev = device()
+    L, n_pages, P, nb = 3, 40, HYBRID12.page_bytes, 128
+    st = torch.empty((L, n_pages * P), dtype=torch.uint8).pin_memory()
+    st.view(torch.int32).random_(generator=torch.Generator().manual_seed(11))
+    cache = torch.full((L, nb * P), POISON, dtype=torch.uint8, device=dev)
+    bt = torch.from_numpy(gen_block_table(12, 0, n_pages, nb)).to(dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_restore_kv_pages(hs.ptr_array([st[l] for l in range(L)], dev),
+                           hs.ptr_array([cache[l] for l in range(L)], dev), L, bt, n_pages, P, nb,
+                           err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    c = cache.view(L, nb, P).cpu()
+    assert torch.equal(c[:, bt.long().cpu()], st.view(L, n_pages, P))
+    mask = torch.ones(nb, dtype=torch.bool)
+    mask[bt.long().cpu()] = False
+    assert bool((c[:, mask] == POISON).all())
