@@ -79,7 +79,7 @@ def kv_bytes(n_layers, n_pages, page_bytes):
     return 2 * n_layers * n_pages * page_bytes
 
 
-KERNEL_OF = {"decode": "gla_recurrent_kernel<128>", "prefill": "gla_chunked_tc_kernel",
+KERNEL_OF = {"decode": "gla_decode_kernel<128>", "prefill": "gla_chunked_tc_kernel",
              "restore": "kv_scatter_kernel+slot_copy_kernel"}
 
 
@@ -259,6 +259,63 @@ class Hybrid12:
                 self.graphs[key + (ph,)] = g
                 self.n_launch[key + (ph,)] = n
         torch.cuda.synchronize(self.dev)
+
+    def capture_steps(self, n):
+        """One CUDA graph per timed step (seed = step index mod seeds) holding the
+        phases of all nine requests, with timing events recorded between phases
+        inside the graph, so a step is one graph launch and the per-phase times are
+        device times of the kernels themselves.  Returns False (nothing captured)
+        where this PyTorch cannot record events inside a graph."""
+        torch = self.torch
+        try:
+            torch.cuda.Event(enable_timing=True, external=True)
+        except TypeError:
+            return False
+        side = torch.cuda.Stream(self.dev)
+        self.step_graphs = []
+        for i in range(n):
+            s = i % self.seeds
+            g = torch.cuda.CUDAGraph()
+            marks, launches = [], 0
+            with torch.cuda.graph(g, stream=side, capture_error_mode="relaxed"):
+                cur = torch.cuda.current_stream(self.dev)
+                prev = torch.cuda.Event(enable_timing=True, external=True)
+                prev.record(cur)
+                for r in range(N_REQ):
+                    for ph in self.PHASES:
+                        nl = getattr(self, "phase_" + ph)(s, r, cur.cuda_stream)
+                        e = torch.cuda.Event(enable_timing=True, external=True)
+                        e.record(cur)
+                        marks.append((ph, self.bytes_of(r, ph), nl, prev, e))
+                        prev = e
+                        launches += nl
+            self.step_graphs.append((s, g, marks, launches))
+        torch.cuda.synchronize(self.dev)
+        return True
+
+    def replay_step(self, i):
+        """Step i from its graph: host alignment of the nine requests, then one
+        graph launch.  Returns the number of kernel launches."""
+        s, g, _, launches = self.step_graphs[i % len(self.step_graphs)]
+        for R in self.req:
+            L = R["L"]
+            c, n_pages, tail = self.hs.hs_align_prefix(
+                L, L, list(range(self.S.ckpt, L + 1, self.S.ckpt)), self.S.page)
+            assert (c, n_pages, tail) == (R["c"], R["n_pages"], TAIL)
+        g.replay()
+        return launches
+
+    def step_phase_times(self):
+        """{phase: [bytes, ms, launches]} from the events inside every step graph
+        (each holds the times of its latest replay)."""
+        out = {}
+        for _, _, marks, _ in self.step_graphs:
+            for ph, nb, nl, e0, e1 in marks:
+                t = out.setdefault(ph, [0, 0.0, 0])
+                t[0] += nb
+                t[1] += e0.elapsed_time(e1)
+                t[2] += nl
+        return out
 
     def bytes_of(self, r, ph):
         R = self.req[r]
@@ -479,8 +536,11 @@ def e2e_run(wl, steps, warmup):
     """Same step with every request's inputs in pinned host memory (KV staging
     pages, checkpoint state, q/k/v/log-gates) copied to the device inside the
     timed region, and its outputs (o, final state, emitted checkpoint) copied
-    back.  Host buffers exist for seed 0; every step uses them."""
-    torch, hs = wl.torch, wl.hs
+    back.  Copies run on their own streams, so request r+1's inputs arrive and
+    request r-1's outputs leave while request r computes; events order every
+    reuse of a device buffer.  Host buffers exist for seed 0; every step uses
+    them."""
+    torch = wl.torch
     dev, stream = wl.dev, wl.stream
     host = []
     h2d = d2h = 0
@@ -491,16 +551,40 @@ def e2e_run(wl, steps, warmup):
         host.append((hb, ob))
         h2d += sum(t.numel() * t.element_size() for t in hb.values())
         d2h += sum(t.numel() * t.element_size() for t in ob.values())
+    s_in = torch.cuda.Stream(dev)
+    s_out = torch.cuda.Stream(dev)
+    ev = lambda: torch.cuda.Event()
+    consumed = [None] * N_REQ     # compute of request r done with its device inputs
+    read = [None] * N_REQ         # device outputs of request r copied to the host
 
     def step():
+        ready = []
         for r in range(N_REQ):
-            hb, ob = host[r]
-            I, O = wl.inp[(0, r)], wl.out[r]
-            for k in hb:
-                I[k].copy_(hb[k], non_blocking=True)
+            hb, _ = host[r]
+            I = wl.inp[(0, r)]
+            if consumed[r] is not None:
+                s_in.wait_event(consumed[r])
+            with torch.cuda.stream(s_in):
+                for k in hb:
+                    I[k].copy_(hb[k], non_blocking=True)
+            e = ev()
+            e.record(s_in)
+            ready.append(e)
+        for r in range(N_REQ):
+            _, ob = host[r]
+            O = wl.out[r]
+            stream.wait_event(ready[r])
+            if read[r] is not None:
+                stream.wait_event(read[r])
             wl.request(0, r, None)
-            for k in ob:
-                ob[k].copy_(O[k], non_blocking=True)
+            consumed[r] = ev()
+            consumed[r].record(stream)
+            s_out.wait_event(consumed[r])
+            with torch.cuda.stream(s_out):
+                for k in ob:
+                    ob[k].copy_(O[k], non_blocking=True)
+            read[r] = ev()
+            read[r].record(s_out)
 
     for _ in range(warmup):
         step()
@@ -508,8 +592,10 @@ def e2e_run(wl, steps, warmup):
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    s_in.wait_stream(stream)        # no copy starts before the timed region
     for _ in range(steps):
         step()
+    stream.wait_stream(s_out)       # ... and the last one ends inside it
     e1.record(stream)
     torch.cuda.synchronize(dev)
     t = e0.elapsed_time(e1) * 1e-3
@@ -817,8 +903,14 @@ def main():
 
     wl = Hybrid12(dev)
     wl.capture()
+    # one graph per timed step (all phases of the nine requests, timing events inside);
+    # per-phase graphs with events around each replay where that is unavailable
+    whole = wl.capture_steps(args.steps)
     for i in range(args.warmup):
-        wl.step(i)
+        if whole:
+            wl.replay_step(i)
+        else:
+            wl.step(i)
     torch.cuda.synchronize(dev)
 
     timer = LaunchTimer(torch, wl.stream)
@@ -831,7 +923,7 @@ def main():
     e0.record(wl.stream)
     launches = 0
     for i in range(args.steps):
-        launches += wl.step(i, timer)
+        launches += wl.replay_step(i) if whole else wl.step(i, timer)
     e1.record(wl.stream)
     torch.cuda.synchronize(dev)
     barrier(ws)
@@ -841,7 +933,7 @@ def main():
     value = aggregate_value(TOKENS_PER_STEP, args.steps, ws, t)
 
     peak, peak_kind = _peaks()
-    groups = timer.summary()
+    groups = wl.step_phase_times() if whole else timer.summary()
     traffic = _traffic()
 
     def roofline(phase):
@@ -866,6 +958,8 @@ def main():
         "roofline": roofline(dominant),
         "roofline_by_phase": {k: roofline(k) for k in groups},
         "gpu_launches": launches,
+        "launch": "one CUDA graph per step, phase events inside the graph" if whole
+                  else "one CUDA graph per request phase, events around each replay",
         "clocks": clk,
     }
     if rank == 0 and not args.no_extras:

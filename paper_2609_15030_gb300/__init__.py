@@ -38,6 +38,7 @@ HS_SHORT_SEGMENT = 8
 HS_LINATTN_AUTO = 0
 HS_LINATTN_RECURRENT = 1
 HS_LINATTN_CHUNKED_TC = 2
+HS_LINATTN_SINGLE_TOKEN = 3
 
 EXPORTED = ("hs_status_string", "hs_version", "hs_align_prefix", "hs_restore_kv_pages",
             "hs_restore_state", "hs_checkpoint_states", "hs_linattn_prefill_from_state",

@@ -61,6 +61,7 @@ constexpr int kShort = 8; // segments of at most this many tokens run token by t
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kFastMinLog2 = -64.0f;      // factorised form if every 2^{Lam_last} >= 2^-64
 constexpr uint64_t kTimeoutNs = 1000000000ull;
+constexpr int kPrefetch = 3;                // segments requested into L2 ahead of the staged one
 
 // shared memory map (offsets from a 1024-byte aligned base).  Every tf32
 // shared-memory operand is K-major (kind::tf32 takes no transposed
@@ -207,6 +208,20 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     uint32_t ph_tma = 0, ph_a = 0, ph_o = 0, ph_s = 0;
     bool aborted = false;
 
+    // L2 prefetch of the 64 tokens from local position t (if any are this problem's)
+    auto prefetch = [&](int64_t t) {
+        if (t >= n)
+            return;
+        const int32_t y = (int32_t)((int64_t)b * p.max_tokens + t);
+        const int32_t x = h * D;
+        tma_prefetch_2d(&maps.q, x, y);
+        tma_prefetch_2d(&maps.k, x, y);
+        tma_prefetch_2d(&maps.v, x, y);
+        tma_prefetch_2d(&maps.g, x, y);
+    };
+    // staged inputs of the segment at local position tok_local; segments after the
+    // first start on the 64-token grid, so the segment kPrefetch ahead starts at
+    // tok_local + 64 * kPrefetch and is requested into L2 now
     auto issue_tma = [&](int64_t tok_local) {
         const int32_t y = (int32_t)((int64_t)b * p.max_tokens + tok_local);
         const int32_t x = h * D;
@@ -216,6 +231,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tma_load_2d(sb + OFF_SV, &maps.v, x, y, bar_tma);
         tma_load_2d(sb + OFF_SG, &maps.g, x, y, bar_tma);
         tma_inflight = true;
+        if (tok_local > 0)
+            prefetch(tok_local + (int64_t)CH * kPrefetch);
     };
     // the issuer waits on an mbarrier, then everyone meets; false if a wait ran out
     auto wait_all = [&](uint32_t bar, uint32_t &ph) -> bool {
@@ -249,8 +266,13 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         return slot + (int64_t)h * D * D;
     };
 
-    if (tid == kIssuer)
+    if (tid == kIssuer) {
         issue_tma(0);
+        // the first kPrefetch segments after the first one
+        const int64_t t1 = min(end, (pos0 / CH + 1) * CH) - pos0;
+        for (int j = 0; j < kPrefetch; ++j)
+            prefetch(t1 + (int64_t)CH * j);
+    }
 
     // incoming state -> TMEM, transposed: S^T[e][d] = state[d][e]
     float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;

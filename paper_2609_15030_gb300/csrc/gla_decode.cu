@@ -1,0 +1,127 @@
+// Gated linear attention, one token per problem (a decode step):
+//     S' = diag(g) S + k v^T,   o = q S',   g = exp(a).
+//
+// One CTA per (problem, head).  Thread (rg, cg) holds rows [16*rg, 16*rg+16)
+// and columns [4*cg, 4*cg+4) of the d x d float32 state in registers; the
+// lanes of a warp are the column groups, so every state load and store of a
+// warp is whole 512-byte rows.  The token's inputs are read straight from
+// global memory (each row group's q/k/a are one broadcast per warp), the state
+// goes back to memory as soon as it is updated, and the row groups' partial
+// outputs meet once in shared memory: one block-wide barrier per step.
+//
+// The arithmetic is exactly that of the per-token recurrent kernel and of the
+// short segments of the chunked tensor-core kernel: g = expf(a); every element
+// becomes fmaf(g_d, S[d][e], k_d * v_e); each group of 16 rows gives a partial
+// dot product by one fma chain in increasing row order; o_e is the left-to-right
+// sum of the group partials.  So the three kernels agree bit for bit.
+#include "hs_internal.cuh"
+
+namespace hs {
+namespace {
+
+__device__ __forceinline__ float bf16_lo(uint32_t w)
+{
+    return __uint_as_float(w << 16);
+}
+
+__device__ __forceinline__ float bf16_hi(uint32_t w)
+{
+    return __uint_as_float(w & 0xFFFF0000u);
+}
+
+template <int D>
+__global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __grid_constant__ GlaParams p)
+{
+    constexpr int NCG = D / 4;        // column groups of 4 (lanes)
+    constexpr int NRG = D / 16;       // row groups of 16
+    __shared__ __align__(16) float spart[NRG][D];
+    const int b = blockIdx.x / p.n_heads;
+    const int h = blockIdx.x - b * p.n_heads;
+    if (p.n_tokens[b] <= 0)
+        return;
+    const int64_t pos0 = p.pos0[b];
+    pdl_wait_and_release();
+    const int tid = threadIdx.x;
+    const int cg = tid % NCG;
+    const int rg = tid / NCG;
+
+    float *st = p.state + ((int64_t)b * p.n_heads + h) * D * D;
+    float4 S[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+        S[r] = *reinterpret_cast<const float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg);
+
+    const int64_t row = ((int64_t)b * p.max_tokens) * p.n_heads + h;   // the call's one token
+    const uint4 *q8 = reinterpret_cast<const uint4 *>(p.q + row * D + 16 * rg);
+    const uint4 *k8 = reinterpret_cast<const uint4 *>(p.k + row * D + 16 * rg);
+    const float4 *a4 = reinterpret_cast<const float4 *>(p.log_g + row * D + 16 * rg);
+    const uint2 v2 = *reinterpret_cast<const uint2 *>(p.v + row * D + 4 * cg);
+    uint32_t qw[8], kw[8];
+    float a[16];
+    *reinterpret_cast<uint4 *>(&qw[0]) = q8[0];
+    *reinterpret_cast<uint4 *>(&qw[4]) = q8[1];
+    *reinterpret_cast<uint4 *>(&kw[0]) = k8[0];
+    *reinterpret_cast<uint4 *>(&kw[4]) = k8[1];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+        *reinterpret_cast<float4 *>(&a[4 * j]) = a4[j];
+    const float4 v4 = make_float4(bf16_lo(v2.x), bf16_hi(v2.x), bf16_lo(v2.y), bf16_hi(v2.y));
+
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+        const float g = expf(a[r]);
+        const float kk = (r & 1) ? bf16_hi(kw[r >> 1]) : bf16_lo(kw[r >> 1]);
+        const float qq = (r & 1) ? bf16_hi(qw[r >> 1]) : bf16_lo(qw[r >> 1]);
+        S[r].x = fmaf(g, S[r].x, kk * v4.x);
+        S[r].y = fmaf(g, S[r].y, kk * v4.y);
+        S[r].z = fmaf(g, S[r].z, kk * v4.z);
+        S[r].w = fmaf(g, S[r].w, kk * v4.w);
+        acc.x = fmaf(qq, S[r].x, acc.x);
+        acc.y = fmaf(qq, S[r].y, acc.y);
+        acc.z = fmaf(qq, S[r].z, acc.z);
+        acc.w = fmaf(qq, S[r].w, acc.w);
+    }
+#pragma unroll
+    for (int r = 0; r < 16; ++r)
+        *reinterpret_cast<float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
+    *reinterpret_cast<float4 *>(&spart[rg][4 * cg]) = acc;
+
+    const int C = p.ckpt_interval;
+    if (C > 0 && p.ckpt_slots != nullptr && (pos0 + 1) % C == 0) {
+        float *slot = p.ckpt_slots[p.ck_base[b]];
+        if (slot == nullptr) {
+            if (tid == 0)
+                report(p.d_err, HS_DEVERR_NULL);
+        } else if ((reinterpret_cast<uintptr_t>(slot) & 15u) != 0) {
+            if (tid == 0)
+                report(p.d_err, HS_DEVERR_MISALIGNED);
+        } else {
+            slot += (int64_t)h * D * D;
+#pragma unroll
+            for (int r = 0; r < 16; ++r)
+                *reinterpret_cast<float4 *>(slot + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
+        }
+    }
+    __syncthreads();
+    // o_e = ((p_0 + p_1) + p_2) + ... over the row groups
+    if (tid < D) {
+        float sum = spart[0][tid];
+#pragma unroll
+        for (int g = 1; g < NRG; ++g)
+            sum += spart[g][tid];
+        p.o[row * D + tid] = sum;
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_gla_decode(const GlaParams &p, int d, cudaStream_t s)
+{
+    const unsigned grid = (unsigned)p.batch * (unsigned)p.n_heads;
+    if (d == 128)
+        return launch_pdl(gla_decode_kernel<128>, dim3(grid), dim3(256), 0, s, p);
+    return launch_pdl(gla_decode_kernel<64>, dim3(grid), dim3(64), 0, s, p);
+}
+
+}  // namespace hs

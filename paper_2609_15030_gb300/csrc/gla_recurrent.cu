@@ -106,6 +106,12 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_recurrent_kernel(const
                 }
             }
         }
+        if (t0 + tb >= n) {
+            // final state out before the output reduction, so the store drains behind it
+#pragma unroll
+            for (int r = 0; r < 16; ++r)
+                *reinterpret_cast<float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
+        }
         __syncthreads();
         for (int idx = tid; idx < tb * D; idx += NTH) {
             const int tt = idx / D, e = idx - (idx / D) * D;
@@ -118,9 +124,6 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_recurrent_kernel(const
         }
         __syncthreads();
     }
-#pragma unroll
-    for (int r = 0; r < 16; ++r)
-        *reinterpret_cast<float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
 }
 
 }  // namespace

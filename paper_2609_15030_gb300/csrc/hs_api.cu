@@ -170,7 +170,7 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
     if (s.batch < 0 || s.n_heads < 1 || s.max_tokens < 0 || s.reserved != 0)
         return HS_ERR_INVALID_ARG;
     if (s.kernel != HS_LINATTN_AUTO && s.kernel != HS_LINATTN_RECURRENT &&
-        s.kernel != HS_LINATTN_CHUNKED_TC)
+        s.kernel != HS_LINATTN_CHUNKED_TC && s.kernel != HS_LINATTN_SINGLE_TOKEN)
         return HS_ERR_INVALID_ARG;
     if (s.d_k != s.d_v || (s.d_k != 64 && s.d_k != 128))
         return HS_ERR_UNSUPPORTED;
@@ -228,16 +228,21 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
     const bool tc_ok = hs::gla_chunked_tc_supported(s.d_k, s.batch, s.max_tokens);
     if (s.kernel == HS_LINATTN_CHUNKED_TC && !tc_ok)
         return HS_ERR_UNSUPPORTED;
-    // AUTO: calls whose tails are all short (decode steps) go to the recurrent kernel,
-    // which computes such segments bit for bit like the chunked kernel does, so the
-    // choice never changes results; everything else takes the tensor-core kernel
     int32_t max_n = 0;
     for (int32_t b = 0; b < s.batch; ++b)
         max_n = n_tokens[b] > max_n ? n_tokens[b] : max_n;
+    if (s.kernel == HS_LINATTN_SINGLE_TOKEN && max_n > 1)
+        return HS_ERR_UNSUPPORTED;
+    // AUTO: decode steps (one token per problem) take the single-token kernel, other calls
+    // whose tails are all short the recurrent kernel; both compute such segments bit for
+    // bit like the chunked kernel does, so the choice never changes results; everything
+    // else takes the tensor-core kernel
     const bool use_tc = s.kernel == HS_LINATTN_CHUNKED_TC ||
                         (s.kernel == HS_LINATTN_AUTO && tc_ok && max_n > HS_SHORT_SEGMENT);
     if (use_tc)
         return cuda_status(hs::launch_gla_chunked_tc(p, s.d_k, stream));
+    if (s.kernel == HS_LINATTN_SINGLE_TOKEN || (s.kernel == HS_LINATTN_AUTO && max_n == 1))
+        return cuda_status(hs::launch_gla_decode(p, s.d_k, stream));
     return cuda_status(hs::launch_gla_recurrent(p, s.d_k, stream));
 }
 

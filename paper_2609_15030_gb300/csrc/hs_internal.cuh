@@ -24,6 +24,13 @@ template <typename... KArgs, typename... Args>
 inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
                               cudaStream_t stream, Args &&...args)
 {
+    // Every kernel of the library asks for the largest shared-memory carveout, so SMs
+    // keep one L1/shared split across back-to-back launches of different kernels
+    // instead of reconfiguring between them (none of them relies on L1 reuse).
+    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                         (int)cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess)
+        return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
@@ -71,6 +78,7 @@ cudaError_t launch_kv_scatter(const void *const *staging, void *const *cache, in
 cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t n,
                              int64_t floats_each, int32_t *d_err, int sm_count, cudaStream_t s);
 cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);
+cudaError_t launch_gla_decode(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s);
 bool gla_chunked_tc_supported(int d, int64_t batch, int64_t max_tokens);
 

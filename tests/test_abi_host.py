@@ -157,6 +157,8 @@ def test_prefill_host_validation():
         (dict(o=FAKE + 4), hs.HS_ERR_MISALIGNED),
         (dict(log_g=FAKE + 8), hs.HS_ERR_MISALIGNED),
         (dict(shape_kw=dict(kernel=7)), hs.HS_ERR_INVALID_ARG),
+        (dict(shape_kw=dict(kernel=hs.HS_LINATTN_SINGLE_TOKEN), n_tokens=[2]),
+         hs.HS_ERR_UNSUPPORTED),                       # the single-token kernel: n_tokens <= 1
     ]
     for kw, code in cases:
         with pytest.raises(hs.HsError) as e:

@@ -284,6 +284,69 @@ def test_short_segments_match_across_kernels():
     _check(*res[0], ro, rS, rck, pos0, n_tok, "short")
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_single_token_steps_match_across_kernels(d):
+    """Decode steps (at most one token per problem): the single-token kernel, the
+    recurrent kernel, the tensor-core kernel's token-by-token path and AUTO agree
+    bit for bit over consecutive steps, including a step that ends on a checkpoint
+    boundary and problems without a token; the result follows the oracle."""
+    dev = device()
+    B, nH, steps, C = 5, 4, 6, 64
+    pos0 = [0, 61, 126, 4093, 700]      # problems 1-3 cross a 64-token boundary in these steps
+    inp = gen_linear(21, d, B, steps, nH, d, d)
+    S0 = gen_state(21, d, B, nH, d, d)
+    kernels = [hs.HS_LINATTN_SINGLE_TOKEN, hs.HS_LINATTN_RECURRENT, hs.HS_LINATTN_AUTO]
+    if d == 128:
+        kernels.append(hs.HS_LINATTN_CHUNKED_TC)
+    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    tok_b, tok_f = nH * d * 2, nH * d * 4
+    res = []
+    for kern in kernels:
+        state = to_dev(np.asarray(S0, np.float32), dev)
+        o = torch.full((B, steps, nH, d), float("nan"), device=dev)
+        slots = torch.full((B * steps, nH, d, d), float("nan"), device=dev)
+        ptrs = hs.ptr_array([slots[i] for i in range(B * steps)], dev)
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+        shape = hs.make_shape(B, nH, d, d, steps, kern)
+        for j in range(steps):
+            n_tok = [0 if (b == 4 and j % 2) else 1 for b in range(B)]   # problem 4: every other step
+            p0 = [pos0[b] + j for b in range(B)]
+            # one checkpoint slot per problem and step (only boundary steps write theirs)
+            base = [b * steps + j for b in range(B)]
+            hs.hs_linattn_prefill_from_state(
+                shape, q.data_ptr() + j * tok_b, k.data_ptr() + j * tok_b,
+                v.data_ptr() + j * tok_b, a.data_ptr() + j * tok_f, o.data_ptr() + j * tok_f,
+                state, p0, n_tok, C, _slots_for(p0, n_tok, C, slots, base, dev), err)
+        torch.cuda.synchronize()
+        assert err.item() == 0
+        res.append((o.cpu().numpy(), state.cpu().numpy(), slots.cpu().numpy()))
+    for o, S, sl in res[1:]:
+        assert np.array_equal(o.view(np.uint32), res[0][0].view(np.uint32))
+        assert np.array_equal(S.view(np.uint32), res[0][1].view(np.uint32))
+        assert np.array_equal(sl.view(np.uint32), res[0][2].view(np.uint32))
+    # oracle: problem 4 sees its tokens 0, 2, 4 (odd steps carry none)
+    o0, S_end, sl0 = res[0]
+    for b in range(B):
+        js = [j for j in range(steps) if not (b == 4 and j % 2)]
+        sub = type(inp)(*(x[b:b + 1, js] for x in (inp.q, inp.k, inp.v, inp.a)))
+        ro, rS, rck = oracle.gla(sub.q, sub.k, sub.v, sub.a, [pos0[b]], [len(js)],
+                                 S0=S0[b:b + 1], C_=C)
+        assert maxnorm_err(o0[b, js], ro[0], axes=(0, 2)) <= TOL
+        assert maxnorm_err(S_end[b:b + 1], rS, axes=(2, 3)) <= TOL
+        jb = [j for j in js if (pos0[b] + j + 1) % C == 0]      # steps ending on the grid
+        assert rck[0].shape[0] == len(jb) == (1 if b in (1, 2, 3) else 0)
+        for m, j in enumerate(jb):
+            assert maxnorm_err(sl0[b * steps + j], rck[0][m], axes=(1, 2)) <= TOL
+
+
+def _slots_for(p0, n_tok, C, slots, base, dev):
+    """Checkpoint-slot array of one call: one entry per checkpoint the call emits, in
+    problem order (the layout hs_linattn_num_checkpoints counts)."""
+    ptrs = [slots[base[b]] for b in range(len(p0))
+            if n_tok[b] and (p0[b] + n_tok[b]) // C - p0[b] // C]
+    return hs.ptr_array(ptrs, dev) if ptrs else None
+
+
 @pytest.mark.parametrize("suffix", [1, 3, 4, 5, 8, 9, 64, 65, 127])
 def test_table4_suffix_lengths_auto_resume_bitwise(suffix):
     """The repaired path recomputes suffixes of 1, 3, 4, 5 and 1,791-1,792 tokens
