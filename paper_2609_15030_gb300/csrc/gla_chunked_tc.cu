@@ -14,35 +14,37 @@
 //
 // One CTA owns one (problem, head) and walks its segments in order; the
 // float32 state lives in tensor memory (TMEM) for the whole call, stored
-// transposed (lane = value dim e, column = key dim d) so that it is directly
-// the A operand of the inter-chunk product.  Per segment:
-//   1. TMA stages q, k, v (bf16) and the log-gates (f32) of 64 tokens;
-//   2. 256 threads build the tf32 operands in 128-byte-swizzled layouts: each
-//      thread scans 32 tokens of one key dimension and the two halves of the
-//      chunk are joined with warp shuffles;
-//   3. one thread issues the MMAs:  D_A = Q~ K~^T;  D_O = S^T Q~^T (A operand
-//      read from TMEM);  D_O += V^T A^T;  S^T += V^T K~  (all kind::tf32 with
-//      K-major operands, fp32 accumulators in TMEM);
-//   4. the causal mask is applied to D_A between the two groups, outputs are
-//      streamed from D_O to global memory, and the state is scaled by
-//      2^{Lam_last} column by column (TMEM -> registers -> TMEM); checkpoint
-//      slots are written from the same registers.
-// The next segment's TMA load is issued as soon as the staging buffers have
-// been consumed, so it overlaps the MMAs and the epilogue.
+// transposed (lane = value dim e, column = key dim d).
 //
-// The factorised form needs 2^{-Lam_j} to stay finite: when some key
-// dimension decays by more than 2^-64 inside one chunk (zero gates, for
-// instance), that chunk computes A elementwise with 2^{Lam_i - Lam_j} <= 1
-// and updates the state as diag(2^{Lam_last}) S + K^^T V with
-// K^_j = k_j 2^{Lam_last - Lam_j}.  The choice depends only on the chunk's
-// own inputs, as does every operation order, so a resumed run reproduces a
-// full recomputation bit for bit when it starts on the chunk grid.
+// Fast chunks run three kind::f16 MMA groups with fp16 operands and float32
+// accumulators:  D_O = S^T Q~^T (A operand: an fp16 copy of S^T in TMEM),
+// D_A = Q~ K~^T, then [D_O | S^T] += V^T [A ; K~^T]^T as one N=192 product
+// (V^T in TMEM).  fp16 keeps the 10-bit mantissa of tf32 but halves the
+// instructions (K = 16 per MMA).  Two operand sets alternate, so while the
+// tensor core runs chunk c the eight operand warps stage chunk c+1 (cumulative
+// decay scan, Q~, K~, K~^T, V^T); the state pass between chunks applies the
+// pending decay 2^{Lam_last}, writes a due checkpoint and refreshes the fp16
+// copy of S^T.  One more warp issues every MMA and TMA copy.
+//
+// A chunk is fast only if every fp16 operand provably stays below 2^15 in
+// magnitude: |q|, |v|, |K~|, the bound 128 max|q| max|k| on |A|, and a bound
+// on |S| carried from the measured state.  Any other chunk (strong decay,
+// huge values) runs the exact path: tf32 operands, the intra-chunk matrix
+// computed elementwise with 2^{Lam_i - Lam_j} <= 1, and the state updated as
+// diag(2^{Lam_last}) S + K^^T V with K^_j = k_j 2^{Lam_last - Lam_j}.  The
+// choice depends only on the chunk's inputs and on the state it starts from,
+// as does every operation order, so a resumed run reproduces a full
+// recomputation bit for bit when it starts on the chunk grid.  Segments of at
+// most 8 tokens run the per-token recurrence with the recurrent kernel's exact
+// operation order.
 //
 // Every wait on an mbarrier is bounded (1 s); on timeout the CTA reports
 // HS_DEVERR_TIMEOUT, waits (bounded) for its own copies and MMAs in flight,
 // frees its TMEM and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include "hs_internal.cuh"
 #include "sm100_ptx.cuh"
@@ -54,73 +56,83 @@ using namespace ptx;
 
 constexpr int D = 128;    // d_k = d_v
 constexpr int CH = 64;    // chunk length (absolute grid)
-constexpr int NW = 256;   // worker threads (warps 0..7): operands and epilogues
+constexpr int NW = 256;   // worker threads (warps 0..7): operands, state passes, epilogues
 constexpr int NT = NW + 32;  // + one warp whose lane 0 issues every MMA and TMA copy
 constexpr int kIssuer = NW;
 constexpr int kShort = 8; // segments of at most this many tokens run token by token
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kFastMinLog2 = -64.0f;      // factorised form if every 2^{Lam_last} >= 2^-64
+constexpr float kF16Lim = 32768.0f;         // fast-path fp16 operands stay below 2^15
 constexpr uint64_t kTimeoutNs = 1000000000ull;
-constexpr int kPrefetch = 3;                // segments requested into L2 ahead of the staged one
+constexpr int kPrefetch = 2;                // segments requested into L2 ahead of the staged one
 
-// shared memory map (offsets from a 1024-byte aligned base).  Every tf32
-// shared-memory operand is K-major (kind::tf32 takes no transposed
-// shared-memory operand); V^T is the A operand of both token-contracting
-// products and lives in tensor memory.
-constexpr uint32_t OFF_QT = 0;          // Q~   [64 tok i][128 d]  tf32, swizzled   32 KiB
-constexpr uint32_t OFF_KT = 32768;      // K~   [64 tok j][128 d]                   32 KiB
-constexpr uint32_t OFF_B2 = 65536;      // [A ; K~^T] [64 i + 128 d][64 tok j]  (K^^T on the exact path)  48 KiB
+// shared memory map (offsets from a 1024-byte aligned base).  Operands are
+// K-major with the 128-byte swizzle.
+constexpr uint32_t SET_BYTES = 57344;   // one fast operand set:
+constexpr uint32_t S_QH = 0;            //   Q~  fp16 [64 tok i][128 d]                 16 KiB
+constexpr uint32_t S_KH = 16384;        //   K~  fp16 [64 tok j][128 d]                 16 KiB
+constexpr uint32_t S_B2H = 32768;       //   [A ; K~^T] fp16 [64 i + 128 d][64 tok j]   24 KiB
+constexpr uint32_t X_QT = 0;            // exact path (over both sets): Q~ tf32 [64][128]     32 KiB
+constexpr uint32_t X_LAM = 32768;       //   Lam f32 [64 tok][128 d], row-major                 32 KiB
+constexpr uint32_t X_B2 = 65536;        //   [A ; K^^T] tf32 [64 i + 128 d][64 tok j]           48 KiB
 constexpr uint32_t OFF_SQ = 114688;     // staged q  bf16 [64][128]                16 KiB
 constexpr uint32_t OFF_SK = 131072;     // staged k                                 16 KiB
 constexpr uint32_t OFF_SV = 147456;     // staged v                                 16 KiB
 constexpr uint32_t OFF_SG = 163840;     // staged log-gates f32 [64][128]           32 KiB
-constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim, one buffer per chunk parity   1 KiB
-constexpr uint32_t OFF_TOT = 197632;    // per-half log2-decay totals [2][128]      1 KiB
-constexpr uint32_t OFF_BAR = 198656;    // 4 mbarriers
-constexpr uint32_t OFF_MISC = 198688;   // TMEM base address, abort flag, exact-path flags (per parity)
-constexpr uint32_t SMEM_BYTES = 198720 + 1024;
+constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim, one buffer per parity   1 KiB
+constexpr uint32_t OFF_TOT = 197632;    // partial log2-decay totals [4 token quarters][128]  2 KiB
+constexpr uint32_t OFF_RED = 199680;    // per warp [8][8]: max |q|, fast-path flag, max |k|, max |v|, max |S|
+constexpr uint32_t OFF_BAR = 199936;    // 4 mbarriers
+constexpr uint32_t OFF_MISC = 199968;   // TMEM base address, abort flag
+constexpr uint32_t SMEM_BYTES = 200000 + 1024;
 constexpr uint32_t STAGE_BYTES = 3 * 16384 + 32768;
-constexpr uint32_t SLAB = 64 * 128;     // one 32-column slab of a 64-row operand
-constexpr uint32_t SLAB_B2 = 192 * 128; // one 32-column slab of the 192-row operand [A ; K~^T]
 
-// tensor memory: the output accumulator D_O alternates between two buffers by chunk
-// parity, placed on either side of S^T so that [D_O0 | S^T] and [S^T | D_O1] are each one
-// N=192 accumulator; V^T alternates likewise.  Even chunks order the 192-row operand as
-// [A ; K~^T], odd chunks as [K~^T ; A].
+// tensor memory: D_O alternates between two buffers by chunk parity, placed on
+// either side of S^T so that [D_O0 | S^T] and [S^T | D_O1] are each one N=192
+// accumulator; even chunks order the 192-row operand as [A ; K~^T], odd ones
+// as [K~^T ; A].
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t TM_O0 = 0;           // D_O of even chunks (lane e, col i), 64 cols
-constexpr uint32_t TM_S = 64;           // S^T  128 lanes x 128 cols
+constexpr uint32_t TM_S = 64;           // S^T  float32, 128 lanes x 128 cols
 constexpr uint32_t TM_O1 = 192;         // D_O of odd chunks
-constexpr uint32_t TM_A = 256;          // D_A  128 lanes x 64 cols (lanes 0..63 used)
-constexpr uint32_t TM_V = 320;          // V^T  2 x 64 cols (lane e, col j)
+constexpr uint32_t TM_SH = 256;         // S^T fp16 copy, two key dims per column      64 cols
+constexpr uint32_t TM_A = 320;          // D_A  128 lanes x 64 cols (lanes 0..63 used)
+constexpr uint32_t TM_V = 384;          // V^T: fast, fp16 pairs 2 x 32 cols; exact, f32 64 cols
 
-constexpr uint32_t IDESC_N64 = idesc_tf32(128, 64, 0, 0);    // M=128, N=64, K-major x K-major
-constexpr uint32_t IDESC_N128 = idesc_tf32(128, 128, 0, 0);  // M=128, N=128
-constexpr uint32_t IDESC_N192 = idesc_tf32(128, 192, 0, 0);  // M=128, N=192
+constexpr uint32_t IDF_N64 = idesc_f16(128, 64);
+constexpr uint32_t IDF_N192 = idesc_f16(128, 192);
+constexpr uint32_t IDT_N64 = idesc_tf32(128, 64, 0, 0);
+constexpr uint32_t IDT_N128 = idesc_tf32(128, 128, 0, 0);
 
 struct TmaMaps {
     CUtensorMap q, k, v, g;
 };
 
-
-// byte offset of element (i, j) of A, stored from row rowA of the 192-row operand
-__device__ __forceinline__ uint32_t a_off(int rowA, int i, int j)
+// byte offset of 16-bit element (row, col) of a K-major operand with `rows` rows
+// (64 columns = 128 bytes per row and slab)
+__device__ __forceinline__ uint32_t h_off(int rows, int row, int col)
 {
-    return (uint32_t)((j >> 5) * SLAB_B2 + (rowA + i) * 128 + ((((j & 31) >> 2) ^ (i & 7)) << 4) +
-                      ((j & 3) << 2));
+    return (uint32_t)((col >> 6) * rows * 128 + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4) +
+                      ((col & 7) << 1));
 }
 
-// 16-byte chunk col4 (tokens 4*col4 .. 4*col4+3) of row d of K~^T, stored from row rowK
-__device__ __forceinline__ uint32_t ktt_chunk(int rowK, int d, int col4)
+// byte offset of 32-bit element (row, col) of a K-major operand (32 columns per slab)
+__device__ __forceinline__ uint32_t t_off(int rows, int row, int col)
 {
-    return (uint32_t)((col4 >> 3) * SLAB_B2 + (rowK + d) * 128 + (((col4 & 7) ^ (d & 7)) << 4));
+    return (uint32_t)((col >> 5) * rows * 128 + row * 128 + ((((col & 31) >> 2) ^ (row & 7)) << 4) +
+                      ((col & 3) << 2));
 }
 
-__device__ __forceinline__ float warp_min(float v)
+// barrier among the eight operand warps only (the MMA-issuing warp does not take part)
+__device__ __forceinline__ void bar_workers()
+{
+    asm volatile("bar.sync 1, 256;" ::: "memory");
+}
+
+__device__ __forceinline__ float warp_max(float v)
 {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
-        v = fminf(v, __shfl_xor_sync(0xffffffffu, v, o));
+        v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
     return v;
 }
 
@@ -129,9 +141,35 @@ __device__ __forceinline__ float bf16f(uint16_t x)
     return __uint_as_float(((uint32_t)x) << 16);
 }
 
+// two floats -> fp16x2 (round to nearest even), the first in the low half
+__device__ __forceinline__ uint32_t pack_h2(float lo, float hi)
+{
+    const __half2 h = __floats2half2_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t *>(&h);
+}
 
+// running elementwise maxima of |x| over fp16 / bf16 pairs (NaN propagates)
+__device__ __forceinline__ __half2 hmax_abs(__half2 acc, uint32_t pair)
+{
+    return __hmax2_nan(acc, __habs2(*reinterpret_cast<const __half2 *>(&pair)));
+}
 
-// 2^x, one MUFU op (relative error ~2^-22; inputs here lie in [-2^7, 2^7])
+__device__ __forceinline__ __nv_bfloat162 bmax_abs(__nv_bfloat162 acc, uint32_t pair)
+{
+    return __hmax2_nan(acc, __habs2(*reinterpret_cast<const __nv_bfloat162 *>(&pair)));
+}
+
+__device__ __forceinline__ float hmax_of(__half2 m)
+{
+    return fmaxf(__low2float(m), __high2float(m));
+}
+
+__device__ __forceinline__ float bmax_of(__nv_bfloat162 m)
+{
+    return fmaxf(__low2float(m), __high2float(m));
+}
+
+// 2^x, one MUFU op (relative error ~2^-22)
 __device__ __forceinline__ float ex2(float x)
 {
     float y;
@@ -143,6 +181,287 @@ __device__ __forceinline__ float ex2(float x)
 __device__ __forceinline__ float rna_tf32(float x)
 {
     return __uint_as_float((__float_as_uint(x) + 0x1000u) & 0xFFFFE000u);
+}
+
+
+// zero the staged rows past a segment of L < 64 tokens (all threads, or the operand
+// warps only)
+__device__ __forceinline__ void zero_tail(uint8_t *smem, int L, bool workers_only)
+{
+    const int tid = threadIdx.x;
+
+    if (L < CH) {
+        const int nthr = workers_only ? NW : NT;
+        for (int idx = tid; idx < (CH - L) * 80; idx += nthr) {
+            const int row = L + idx / 80, c = idx % 80;
+            uint4 *dst;
+            if (c < 16)
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SQ + row * 256) + c;
+            else if (c < 32)
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SK + row * 256) + (c - 16);
+            else if (c < 48)
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SV + row * 256) + (c - 32);
+            else
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SG + row * 512) + (c - 48);
+            *dst = make_uint4(0u, 0u, 0u, 0u);
+        }
+        if (workers_only)
+            bar_workers();
+        else
+            __syncthreads();
+    }
+}
+
+
+// ---- fast operands of a staged long segment into set `par`.  Thread (dp, qt) owns key
+// dims 2dp, 2dp+1 for tokens [16 qt, 16 qt + 16): it sums their log2-gates, then runs
+// the cumulative sum again from the earlier quarters' totals (shared memory;
+// 2^{Lam_last} into gam[par]) while it writes
+// Q~ and K~ (token-major, the d-contractions' operands) and K~^T (rows of [A ; K~^T]),
+// fp16, with 4- and 16-byte stores.  Then thread (e, half) packs V^T into TMEM.  Per
+// warp: max |q|, |k|, |v| and whether every operand fits fp16 (for the guard).
+__device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, int par)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bool worker = warp < 8;
+    const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
+    const int colhalf = warp >> 2;
+    const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
+    const int th = colhalf;
+    const uint16_t *sQ = reinterpret_cast<const uint16_t *>(smem + OFF_SQ);
+    const uint16_t *sK = reinterpret_cast<const uint16_t *>(smem + OFF_SK);
+    const uint16_t *sV = reinterpret_cast<const uint16_t *>(smem + OFF_SV);
+    const float *sG = reinterpret_cast<const float *>(smem + OFF_SG);
+    float *sTot = reinterpret_cast<float *>(smem + OFF_TOT);
+    float *sGam = reinterpret_cast<float *>(smem + OFF_GAM);
+    float *sRed = reinterpret_cast<float *>(smem + OFF_RED);
+
+    if (!worker)
+        return;
+    zero_tail(smem, L, true);
+    const int dp = tid & 63, qt = (tid >> 6) & 3;
+    float amax = -INFINITY;
+    {
+        // quarter totals
+        float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+        for (int x = 0; x < 16; ++x) {
+            const float2 a = *reinterpret_cast<const float2 *>(sG + (16 * qt + x) * D + 2 * dp);
+            amax = fmaxf(amax, fmaxf(a.x, a.y));
+            r0 = fmaf(a.x, kLog2e, r0);
+            r1 = fmaf(a.y, kLog2e, r1);
+        }
+        *reinterpret_cast<float2 *>(sTot + qt * D + 2 * dp) = make_float2(r0, r1);
+    }
+    bar_workers();
+    // the running sums start from the earlier quarters' totals
+    float run0 = 0.f, run1 = 0.f;
+    {
+        float t0 = 0.f, t1 = 0.f;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const float2 t = *reinterpret_cast<const float2 *>(sTot + u * D + 2 * dp);
+            if (u < qt) {
+                run0 += t.x;
+                run1 += t.y;
+            }
+            t0 += t.x;
+            t1 += t.y;
+        }
+        if (qt == 0)
+            *reinterpret_cast<float2 *>(sGam + par * D + 2 * dp) = make_float2(ex2(t0), ex2(t1));
+    }
+    uint8_t *set = smem + par * SET_BYTES;
+    const int rowK = par ? 0 : 64;
+    __nv_bfloat162 bq = __float2bfloat162_rn(0.f), bk = bq;   // max |q|, |k|
+    __half2 hq = __float2half2_rn(0.f), hk = hq;                 // max |Q~|, |K~| (fp16)
+    // two groups of 8 tokens; within a group, token pairs: Q~ and K~ as fp16 pairs of key
+    // dims, K~^T rows 2dp and 2dp+1 as fp16 pairs of tokens (byte permutes of the K~ pairs)
+#pragma unroll 1
+    for (int grp = 0; grp < 2; ++grp) {
+        uint32_t kt0[4], kt1[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            uint32_t kp[2];
+#pragma unroll
+            for (int t = 0; t < 2; ++t) {
+                const int i = 16 * qt + 8 * grp + 2 * u + t;
+                const float2 a = *reinterpret_cast<const float2 *>(sG + i * D + 2 * dp);
+                run0 = fmaf(a.x, kLog2e, run0);
+                run1 = fmaf(a.y, kLog2e, run1);
+                const uint32_t q2 = *reinterpret_cast<const uint32_t *>(sQ + i * D + 2 * dp);
+                const uint32_t k2 = *reinterpret_cast<const uint32_t *>(sK + i * D + 2 * dp);
+                const float q0 = __uint_as_float(q2 << 16), q1 = __uint_as_float(q2 & 0xFFFF0000u);
+                const float k0 = __uint_as_float(k2 << 16), k1 = __uint_as_float(k2 & 0xFFFF0000u);
+                const uint32_t qp = pack_h2(q0 * ex2(run0), q1 * ex2(run1));
+                kp[t] = pack_h2(k0 * ex2(-run0), k1 * ex2(-run1));
+                *reinterpret_cast<uint32_t *>(set + S_QH + h_off(64, i, 2 * dp)) = qp;
+                *reinterpret_cast<uint32_t *>(set + S_KH + h_off(64, i, 2 * dp)) = kp[t];
+                bq = bmax_abs(bq, q2);
+                bk = bmax_abs(bk, k2);
+                hq = hmax_abs(hq, qp);
+                hk = hmax_abs(hk, kp[t]);
+            }
+            kt0[u] = __byte_perm(kp[0], kp[1], 0x5410);   // key dim 2dp: tokens (2u, 2u+1)
+            kt1[u] = __byte_perm(kp[0], kp[1], 0x7632);   // key dim 2dp+1
+        }
+        const int j0 = 16 * qt + 8 * grp;
+        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowK + 2 * dp, j0)) =
+            make_uint4(kt0[0], kt0[1], kt0[2], kt0[3]);
+        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowK + 2 * dp + 1, j0)) =
+            make_uint4(kt1[0], kt1[1], kt1[2], kt1[3]);
+    }
+    // V^T: thread (e, half) packs tokens [32 half, 32 half + 32) of value dim e
+    __nv_bfloat162 bv = __float2bfloat162_rn(0.f);
+    {
+        uint32_t vpk[16];
+#pragma unroll
+        for (int m = 0; m < 16; ++m) {
+            const int i = 32 * th + 2 * m;
+            const uint32_t w = (uint32_t)sV[i * D + e_own] | ((uint32_t)sV[(i + 1) * D + e_own] << 16);
+            bv = bmax_abs(bv, w);
+            vpk[m] = pack_h2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+        }
+        tmem_st16(tmem + lrow + TM_V + 32 * par + 16 * th, vpk);
+    }
+    float mq = warp_max(bmax_of(bq));
+    float mk = warp_max(bmax_of(bk));
+    float mv = warp_max(bmax_of(bv));
+    // non-increasing Lam (|Q~| <= |q|, |A| <= 128 max|q| max|k|) and every fp16 operand
+    // below 2^15; NaN fails
+    bool ok = amax <= 0.f && hmax_of(hq) < kF16Lim && hmax_of(hk) < kF16Lim && mv < kF16Lim;
+    ok = __all_sync(0xffffffffu, ok);
+    if (lane == 0) {
+        sRed[warp * 8 + 0] = mq;
+        sRed[warp * 8 + 1] = ok ? 1.f : 0.f;
+        sRed[warp * 8 + 2] = mk;
+        sRed[warp * 8 + 3] = mv;
+    }
+    tmem_wait_st();
+}
+
+
+// ---- state pass: decay by gam[gpar] (gpar < 0: none), checkpoint slot, fp16 copy of
+// S^T for the next S^T Q~^T, and the largest |S|
+__device__ __forceinline__ void state_pass(uint8_t *smem, uint32_t tmem, int gpar, float *slot, bool copy)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bool worker = warp < 8;
+    const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
+    const int colhalf = warp >> 2;
+    const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
+    const float *sGam = reinterpret_cast<const float *>(smem + OFF_GAM);
+    float *sRed = reinterpret_cast<float *>(smem + OFF_RED);
+
+    if (!worker)
+        return;
+    const int db = colhalf * 64;
+    float r[64];
+    tmem_ld32(tmem + lrow + TM_S + db, *reinterpret_cast<float(*)[32]>(&r[0]));
+    tmem_ld32(tmem + lrow + TM_S + db + 32, *reinterpret_cast<float(*)[32]>(&r[32]));
+    tmem_wait_ld();
+    if (gpar >= 0) {
+        const float *gam = sGam + gpar * D + db;
+#pragma unroll
+        for (int c = 0; c < 16; ++c) {
+            const float4 g4 = *reinterpret_cast<const float4 *>(gam + 4 * c);
+            r[4 * c] *= g4.x;
+            r[4 * c + 1] *= g4.y;
+            r[4 * c + 2] *= g4.z;
+            r[4 * c + 3] *= g4.w;
+        }
+        tmem_st32(tmem + lrow + TM_S + db, *reinterpret_cast<float(*)[32]>(&r[0]));
+        tmem_st32(tmem + lrow + TM_S + db + 32, *reinterpret_cast<float(*)[32]>(&r[32]));
+    }
+    if (slot != nullptr) {
+#pragma unroll
+        for (int x = 0; x < 64; ++x)
+            slot[(int64_t)(db + x) * D + e_own] = r[x];
+    }
+    float m;
+    if (copy) {
+        // the fp16 copy, two key dims per column; its largest magnitude (inf past fp16)
+        __half2 hm = __float2half2_rn(0.f);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            uint32_t u[16];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                u[c] = pack_h2(r[32 * hh + 2 * c], r[32 * hh + 2 * c + 1]);
+                hm = hmax_abs(hm, u[c]);
+            }
+            tmem_st16(tmem + lrow + TM_SH + db / 2 + 16 * hh, u);
+        }
+        m = hmax_of(hm);
+    } else {
+        m = 0.f;
+#pragma unroll
+        for (int x = 0; x < 64; ++x)
+            m = fmaxf(m, fabsf(r[x]));
+    }
+    tmem_wait_st();
+    m = warp_max(m);
+    if (lane == 0)
+        sRed[warp * 8 + 4] = m;
+}
+
+
+// ---- the causally masked intra-chunk matrix A (D_A) -> rows rowA.. of set par's [A ; K~^T]
+__device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
+{
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool worker = warp < 8;
+    const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
+
+    if (!(worker && (warp & 3) < 2))
+        return;
+    const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
+    const int jb = (warp >> 2) * 32;            // this warp's 32 key columns
+    const int rowA = par ? 128 : 0;
+    float r[32];
+    tmem_ld32(tmem + lrow + TM_A + jb, r);
+    tmem_wait_ld();
+    uint8_t *set = smem + par * SET_BYTES;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        uint32_t w[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int j0 = jb + 8 * c + 2 * u;
+            w[u] = pack_h2(j0 <= i ? r[8 * c + 2 * u] : 0.f, j0 + 1 <= i ? r[8 * c + 2 * u + 1] : 0.f);
+        }
+        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowA + i, jb + 8 * c)) =
+            make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+
+// ---- output epilogue of a processed segment: D_O buffer `par` -> o (lane e, 32 rows)
+__device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t tstride, int L, int par)
+{
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const bool worker = warp < 8;
+    const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
+    const int colhalf = warp >> 2;
+    const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
+
+    if (!worker)
+        return;
+    float r[32];
+    const int ib = colhalf * 32;
+    tmem_ld32(tmem + lrow + (par ? TM_O1 : TM_O0) + ib, r);
+    tmem_wait_ld();
+    float *op = ob + (int64_t)ib * tstride + e_own;
+    if (L == CH) {
+#pragma unroll
+        for (int x = 0; x < 32; ++x)
+            __stcs(op + (int64_t)x * tstride, r[x]);
+    } else {
+#pragma unroll
+        for (int x = 0; x < 32; ++x)
+            if (ib + x < L)
+                __stcs(op + (int64_t)x * tstride, r[x]);
+    }
 }
 
 __global__ void __launch_bounds__(NT, 1)
@@ -157,6 +476,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     const uint16_t *sV = reinterpret_cast<const uint16_t *>(smem + OFF_SV);
     float *sG = reinterpret_cast<float *>(smem + OFF_SG);
     float *sTot = reinterpret_cast<float *>(smem + OFF_TOT);
+    float *sGam = reinterpret_cast<float *>(smem + OFF_GAM);
+    float *sRed = reinterpret_cast<float *>(smem + OFF_RED);
     volatile uint32_t *sMisc = reinterpret_cast<volatile uint32_t *>(smem + OFF_MISC);
     const uint32_t bar_tma = sb + OFF_BAR, bar_a = sb + OFF_BAR + 8, bar_o = sb + OFF_BAR + 16,
                    bar_s = sb + OFF_BAR + 24;
@@ -194,17 +515,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // operand-building map: worker owns key dim d = e_own for tokens [32*th, 32*th+32)
     const int d = e_own;
     const int th = colhalf;
-    uint32_t nat[8];       // byte offset of (row 32*th + r, col d) in a 64-row operand
-    {
-        const uint32_t base = (uint32_t)((warp & 3) * SLAB + (32 * th) * 128 + ((lane & 3) << 2));
-        const int cd = lane >> 2;
-#pragma unroll
-        for (int r = 0; r < 8; ++r)
-            nat[r] = base + r * 128 + ((uint32_t)(cd ^ r) << 4);
-    }
 
-    // issuer bookkeeping (lane 0 of warp 8) of work in flight, for the abort path
-    bool tma_inflight = false;
+    // issuer bookkeeping (lane 0 of warp 8) of copies issued, for the abort path
+    uint32_t n_tma = 0;
     uint32_t ph_tma = 0, ph_a = 0, ph_o = 0, ph_s = 0;
     bool aborted = false;
 
@@ -230,7 +543,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tma_load_2d(sb + OFF_SK, &maps.k, x, y, bar_tma);
         tma_load_2d(sb + OFF_SV, &maps.v, x, y, bar_tma);
         tma_load_2d(sb + OFF_SG, &maps.g, x, y, bar_tma);
-        tma_inflight = true;
+        ++n_tma;
         if (tok_local > 0)
             prefetch(tok_local + (int64_t)CH * kPrefetch);
     };
@@ -247,11 +560,25 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
         return true;
     };
-    auto wait_tma = [&]() -> bool {
-        const bool ok = wait_all(bar_tma, ph_tma);
-        if (tid == kIssuer)
-            tma_inflight = false;
-        return ok;
+    auto wait_tma = [&]() -> bool { return wait_all(bar_tma, ph_tma); };
+    // one operand thread waits, then the operand warps meet; the issuer only follows the
+    // phase.  A timeout is seen by everyone at the next sync_all.
+    auto wait_w = [&](uint32_t bar, uint32_t &ph) {
+        if (tid == 0 && !mbar_wait_bounded(bar, ph, kTimeoutNs))
+            sMisc[1] = 1;
+        if (worker) {
+            bar_workers();
+            tc_fence_after();
+        }
+        ph ^= 1;
+    };
+    auto sync_all = [&]() -> bool {
+        __syncthreads();
+        if (sMisc[1]) {
+            aborted = true;
+            return false;
+        }
+        return true;
     };
     auto seg_len = [&](int64_t at) -> int { return (int)(min(end, (at / CH + 1) * CH) - at); };
     auto ckpt_slot = [&](int64_t seg_end) -> float * {
@@ -265,41 +592,57 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
         return slot + (int64_t)h * D * D;
     };
+    // largest |S| recorded by the last state pass (valid after the barrier that follows it)
+    auto state_max = [&]() -> float {
+        float m = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w)
+            m = fmaxf(m, sRed[w * 8 + 4]);
+        return m;
+    };
 
-    if (tid == kIssuer) {
+    if (tid == kIssuer)
         issue_tma(0);
-        // the first kPrefetch segments after the first one
+
+    // incoming state -> TMEM, transposed: S^T[e][d] = state[d][e]; its largest magnitude
+    float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
+    if (worker) {
+        float r[32];
+        float m = 0.f;
+#pragma unroll
+        for (int c0 = 0; c0 < 64; c0 += 32) {
+            const int d0 = colhalf * 64 + c0;
+#pragma unroll
+            for (int x = 0; x < 32; ++x) {
+                r[x] = st_g[(int64_t)(d0 + x) * D + e_own];
+                m = fmaxf(m, fabsf(r[x]));
+            }
+            tmem_st32(tmem + lrow + TM_S + d0, r);
+        }
+        tmem_wait_st();
+        m = warp_max(m);
+        if (lane == 0)
+            sRed[warp * 8 + 4] = m;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (tid == kIssuer) {
+        // the first kPrefetch segments after the first one, once the state is in: the
+        // state and the first segment are not queued behind them
         const int64_t t1 = min(end, (pos0 / CH + 1) * CH) - pos0;
         for (int j = 0; j < kPrefetch; ++j)
             prefetch(t1 + (int64_t)CH * j);
     }
 
-    // incoming state -> TMEM, transposed: S^T[e][d] = state[d][e]
-    float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
-    if (worker) {
-        float r[32];
-#pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 32) {
-            const int d0 = colhalf * 64 + c0;
-#pragma unroll
-            for (int x = 0; x < 32; ++x)
-                r[x] = st_g[(int64_t)(d0 + x) * D + e_own];
-            tmem_st32(tmem + lrow + TM_S + d0, r);
-        }
-        tmem_wait_st();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-
-    // ---- a short segment (<= kShort tokens, staged inputs already waited for): the
-    // per-token recurrence with the recurrent kernel's exact operation order (fma chains
-    // over groups of 16 key rows, group partials summed left to right)
+    // ---- a short segment (<= kShort tokens, staged inputs already waited for, no decay
+    // pending): the per-token recurrence with the recurrent kernel's exact operation order
+    // (fma chains over groups of 16 key rows, group partials summed left to right)
     auto short_segment = [&](int64_t tok_s, int L, int64_t seg_end) {
         for (int idx = tid; idx < L * D; idx += NT)
             sG[idx] = expf(sG[idx]);
         __syncthreads();
-        float *part = reinterpret_cast<float *>(smem + OFF_QT);   // [kShort][8 groups][128]
+        float *part = reinterpret_cast<float *>(smem);   // [kShort][8 groups][128] in the operand sets
         float *slot = ckpt_slot(seg_end);
         if (worker) {
             float S[64];
@@ -322,11 +665,16 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             tmem_st32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
             tmem_st32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
-            if (slot != nullptr) {
+            float m = 0.f;
 #pragma unroll
-                for (int r = 0; r < 64; ++r)
+            for (int r = 0; r < 64; ++r) {
+                m = fmaxf(m, fabsf(S[r]));
+                if (slot != nullptr)
                     slot[(int64_t)(colhalf * 64 + r) * D + e_own] = S[r];
             }
+            m = warp_max(m);
+            if (lane == 0)
+                sRed[warp * 8 + 4] = m;
             tmem_wait_st();
         }
         fence_proxy_async_smem();
@@ -347,117 +695,149 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tc_fence_after();
     };
 
-    // ---- prep of a long segment (staged inputs already waited for): zero the staged rows
-    // past the segment, cumulative log2-gates (per-thread scan of 32 tokens, halves joined
-    // through shared memory, path vote by a warp-shuffle min), Q~ into shared memory and
-    // V^T into tensor memory buffer `par`.  Leaves lam[] in registers.
-    float lam[32];
-    float last = 0.f;
-    auto prep = [&](int L, int par) {
-        if (L < CH) {
-            for (int idx = tid; idx < (CH - L) * 80; idx += NT) {
-                const int row = L + idx / 80, c = idx % 80;
-                uint4 *dst;
-                if (c < 16)
-                    dst = reinterpret_cast<uint4 *>(smem + OFF_SQ + row * 256) + c;
-                else if (c < 32)
-                    dst = reinterpret_cast<uint4 *>(smem + OFF_SK + row * 256) + (c - 16);
-                else if (c < 48)
-                    dst = reinterpret_cast<uint4 *>(smem + OFF_SV + row * 256) + (c - 32);
-                else
-                    dst = reinterpret_cast<uint4 *>(smem + OFF_SG + row * 512) + (c - 48);
-                *dst = make_uint4(0u, 0u, 0u, 0u);
+
+
+
+
+
+    // the guard of a built fast segment (after the barrier that follows build_fast): log-gates
+    // <= 0, and every fp16 operand (Q~, K~, V, A, the fp16 copy of the state it starts
+    // from) below 2^15 in magnitude
+    float mk_cur = 0.f, mv_cur = 0.f;   // maxima |k|, |v| of the pending fast segment
+    float mk_new = 0.f, mv_new = 0.f;
+    auto guard = [&](float s_bound) -> bool {
+        float mq = 0.f, mk = 0.f, mv = 0.f;
+        bool ok = true;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) {
+            mq = fmaxf(mq, sRed[w * 8 + 0]);
+            ok = ok && sRed[w * 8 + 1] != 0.f;
+            mk = fmaxf(mk, sRed[w * 8 + 2]);
+            mv = fmaxf(mv, sRed[w * 8 + 3]);
+        }
+        mk_new = mk;
+        mv_new = mv;
+        return ok && 128.0f * mq * mk < kF16Lim && s_bound < kF16Lim;
+    };
+
+    // ---- one exact segment, from staged inputs, no decay pending and no MMA in flight;
+    // leaves the final state in TMEM, writes its outputs and checkpoint
+    auto exact_segment = [&](int64_t tok_s, int L, int par, int64_t seg_end) -> bool {
+        // cumulative log2-gates: key dim d over 32 tokens per thread, halves joined through
+        // shared memory; 2^{Lam_last} into gam[par]
+        float lam[32];
+        float last = 0.f;
+        zero_tail(smem, L, false);
+        {
+            float run = 0.f;
+            if (worker) {
+#pragma unroll
+                for (int x = 0; x < 32; ++x) {
+                    run = fmaf(sG[(32 * th + x) * D + d], kLog2e, run);
+                    lam[x] = run;
+                }
+                sTot[th * D + d] = run;
             }
             __syncthreads();
-        }
-        float run = 0.f;
-        if (worker) {
+            if (worker) {
+                const float tot0 = sTot[d];
+                last = tot0 + sTot[D + d];   // Lam_last of key dim d
+                if (th) {
 #pragma unroll
-            for (int x = 0; x < 32; ++x) {
-                run = fmaf(sG[(32 * th + x) * D + d], kLog2e, run);
-                lam[x] = run;
+                    for (int x = 0; x < 32; ++x)
+                        lam[x] = tot0 + lam[x];
+                } else {
+                    sGam[par * D + d] = ex2(last);
+                }
             }
-            sTot[th * D + d] = run;
         }
-        if (tid == 0)
-            sMisc[2 + par] = 0;   // exact-path flag of this segment
-        __syncthreads();
         if (worker) {
-            const float tot0 = sTot[d];
-            last = tot0 + sTot[D + d];   // Lam_last of key dim d
-            if (th) {
-#pragma unroll
-                for (int x = 0; x < 32; ++x)
-                    lam[x] = tot0 + lam[x];
-            } else {
-                reinterpret_cast<float *>(smem + OFF_GAM)[par * D + d] = ex2(last);
-            }
-            const float wmin = warp_min(last);
-            if (lane == 0 && wmin < kFastMinLog2)
-                sMisc[2 + par] = 1;
+            // Q~ = q 2^{Lam} (tf32), K^^T = k 2^{Lam_last - Lam} (tf32, rows 64.. of X_B2),
+            // Lam token-major for the elementwise A, V^T float32 into TMEM
             float vtr[32];
 #pragma unroll
-            for (int x = 0; x < 32; ++x) {
-                const int i = 32 * th + x;
-                const float qv = bf16f(sQ[i * D + d]);
-                vtr[x] = bf16f(sV[i * D + d]);
-                *reinterpret_cast<float *>(smem + OFF_QT + nat[x & 7] + (x >> 3) * 1024) =
-                    rna_tf32(qv * ex2(lam[x]));
+            for (int g = 0; g < 8; ++g) {
+                float4 w;
+                float *wv = &w.x;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int x = 4 * g + u;
+                    const int i = 32 * th + x;
+                    *reinterpret_cast<float *>(smem + X_QT + t_off(64, i, d)) =
+                        rna_tf32(bf16f(sQ[i * D + d]) * ex2(lam[x]));
+                    wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam[x]));
+                    reinterpret_cast<float *>(smem + X_LAM)[i * D + d] = lam[x];
+                    vtr[x] = bf16f(sV[i * D + d]);
+                }
+                *reinterpret_cast<float4 *>(smem + X_B2 + t_off(192, 64 + d, 32 * th + 4 * g)) = w;
             }
-            tmem_st32(tmem + lrow + TM_V + 64 * par + 32 * th, vtr);
+            tmem_st32(tmem + lrow + TM_V + 32 * th, vtr);
             tmem_wait_st();
         }
         fence_proxy_async_smem();
-    };
-
-    // ---- output epilogue of a processed segment: D_O buffer `par` -> o (lane e, 32 rows)
-    auto out_epilogue = [&](int64_t tok_s, int L, int par) {
-        if (!worker)
-            return;
-        float r[32];
-        const int ib = colhalf * 32;
-        tmem_ld32(tmem + lrow + (par ? TM_O1 : TM_O0) + ib, r);
-        tmem_wait_ld();
-        float *op = p.o + (((int64_t)b * p.max_tokens + tok_s + ib) * p.n_heads + h) * D + e_own;
-        if (L == CH) {
+        tc_fence_before();
+        __syncthreads();
+        const uint32_t tm_o = par ? TM_O1 : TM_O0;
+        if (tid == kIssuer) {
+            // S^T Q~^T into D_O (A operand: the float32 state in TMEM)
+            tc_fence_after();
 #pragma unroll
-            for (int x = 0; x < 32; ++x)
-                __stcs(op + (int64_t)x * tstride, r[x]);
-        } else {
-#pragma unroll
-            for (int x = 0; x < 32; ++x)
-                if (ib + x < L)
-                    __stcs(op + (int64_t)x * tstride, r[x]);
-        }
-    };
-
-    // ---- state decay by 2^{Lam_last} (buffer `par`), checkpoint from the same registers
-    auto decay_state = [&](int par, float *slot) {
-        if (!worker)
-            return;
-        const float *gam = reinterpret_cast<const float *>(smem + OFF_GAM) + par * D;
-#pragma unroll
-        for (int c0 = 0; c0 < 64; c0 += 32) {
-            const int d0 = colhalf * 64 + c0;
-            float r[32];
-            tmem_ld32(tmem + lrow + TM_S + d0, r);
-            tmem_wait_ld();
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-                const float4 g4 = *reinterpret_cast<const float4 *>(gam + d0 + 4 * c);
-                r[4 * c] *= g4.x;
-                r[4 * c + 1] *= g4.y;
-                r[4 * c + 2] *= g4.z;
-                r[4 * c + 3] *= g4.w;
-            }
-            tmem_st32(tmem + lrow + TM_S + d0, r);
-            if (slot != nullptr) {
-#pragma unroll
-                for (int x = 0; x < 32; ++x)
-                    slot[(int64_t)(d0 + x) * D + e_own] = r[x];
+            for (int kk = 0; kk < D / 8; ++kk) {
+                const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
+                mma_tf32_ts(tmem + tm_o, tmem + TM_S + kk * 8, sdesc_sw128(sb + X_QT + koff, 16, 1024),
+                            IDT_N64, kk > 0);
             }
         }
-        tmem_wait_st();
+        // A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}, j <= i < L, elementwise
+        {
+            const float *lg = reinterpret_cast<const float *>(smem + X_LAM);
+            for (int idx = tid; idx < CH * CH; idx += NT) {
+                const int i = idx >> 6, j = idx & 63;
+                float acc = 0.f;
+                if (j <= i && i < L) {
+                    for (int dd = 0; dd < D; ++dd)
+                        acc = fmaf(bf16f(sQ[i * D + dd]) * bf16f(sK[j * D + dd]),
+                                   ex2(lg[i * D + dd] - lg[j * D + dd]), acc);
+                }
+                *reinterpret_cast<float *>(smem + X_B2 + t_off(192, i, j)) = rna_tf32(acc);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == kIssuer) {
+            tc_fence_after();
+#pragma unroll
+            for (int kk = 0; kk < CH / 8; ++kk) {
+                const uint32_t koff = (kk >> 2) * (192 * 128) + (kk & 3) * 32;
+                mma_tf32_ts(tmem + tm_o, tmem + TM_V + kk * 8, sdesc_sw128(sb + X_B2 + koff, 16, 1024),
+                            IDT_N64, 1);
+            }
+            tc_commit(bar_o);
+        }
+        if (!wait_all(bar_o, ph_o))
+            return false;
+        state_pass(smem, tmem, par, nullptr, false);          // S <- diag(2^{Lam_last}) S
+        tc_fence_before();
+        __syncthreads();
+        if (tid == kIssuer) {
+            tc_fence_after();
+#pragma unroll
+            for (int kk = 0; kk < CH / 8; ++kk) {
+                const uint32_t koff = (kk >> 2) * (192 * 128) + (kk & 3) * 32 + 64 * 128;
+                mma_tf32_ts(tmem + TM_S, tmem + TM_V + kk * 8, sdesc_sw128(sb + X_B2 + koff, 16, 1024),
+                            IDT_N128, 1);
+            }
+            tc_commit(bar_s);
+        }
+        if (!wait_all(bar_s, ph_s))
+            return false;
+        state_pass(smem, tmem, -1, ckpt_slot(seg_end), false);   // checkpoint and |S| of the final state
+        out_epilogue(tmem, p.o + (((int64_t)b * p.max_tokens + tok_s) * p.n_heads + h) * D, tstride, L, par);
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        return true;
     };
 
     int64_t pos = pos0, tok = 0;
@@ -470,203 +850,144 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         pos += seg_len(pos);
     }
 
-    // ---- pipelined long segments
-    if (pos < end && seg_len(pos) > kShort) {
-        if (!wait_tma())
-            goto finish;
-        prep(seg_len(pos), 0);
+    // ---- long segments: fast ones pipelined two deep, exact ones one at a time
+    {
+        const auto out_of = [&](int64_t t) {
+            return p.o + (((int64_t)b * p.max_tokens + t) * p.n_heads + h) * D;
+        };
         int par = 0;
-        bool prev_valid = false;
-        int64_t tok_prev = 0;
-        int L_prev = 0;
-        while (true) {
+        bool have_prep = false, prep_fast = false, qk_issued = false;
+        bool pend = false;
+        int pend_par = 0, pend_L = 0;
+        int64_t pend_tok = 0, pend_end = 0;
+        while (pos < end && seg_len(pos) > kShort) {
             const int L = seg_len(pos);
             const int64_t seg_end = pos + L;
             const bool has_next = seg_end < end;
-            const int L_next = has_next ? seg_len(seg_end) : 0;
-            const bool next_long = has_next && L_next > kShort;
-            const uint32_t rowA = par ? 128u : 0u, rowK = par ? 0u : 64u;
-            const uint32_t tm_o = par ? TM_O1 : TM_O0;
-
-            // Q~ / V^T of this segment and the previous decay are complete
-            tc_fence_before();
-            __syncthreads();
-            const bool slow = sMisc[2 + par] != 0;
-            if (tid == kIssuer) {
-                // S^T Q~^T into D_O[par] (A operand read from tensor memory)
-                tc_fence_after();
-#pragma unroll
-                for (int kk = 0; kk < D / 8; ++kk) {
-                    const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
-                    mma_tf32_ts(tmem + tm_o, tmem + TM_S + kk * 8,
-                                sdesc_sw128(sb + OFF_QT + koff, 16, 1024), IDESC_N64, kk > 0);
-                }
-            }
-            if (worker) {
-                if (!slow) {
-                    // K~ token-major (operand of Q~ K~^T) and transposed (state update)
-#pragma unroll
-                    for (int g = 0; g < 8; ++g) {
-                        float4 kt4;
-                        float *kv4 = &kt4.x;
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const int x = 4 * g + u;
-                            const int i = 32 * th + x;
-                            kv4[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(-lam[x]));
-                            *reinterpret_cast<float *>(smem + OFF_KT + nat[x & 7] + (x >> 3) * 1024) = kv4[u];
-                        }
-                        *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(rowK, d, 8 * th + g)) = kt4;
-                    }
-                } else {
-                    // exact path: K^ = k 2^{Lam_last - Lam} (transposed), cumulative log2-gates
-                    // token-major in the (unused) K~ buffer
-#pragma unroll
-                    for (int g = 0; g < 8; ++g) {
-                        float4 w;
-                        float *wv = &w.x;
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const int x = 4 * g + u;
-                            const int i = 32 * th + x;
-                            wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam[x]));
-                            reinterpret_cast<float *>(smem + OFF_KT)[i * D + d] = lam[x];
-                        }
-                        *reinterpret_cast<float4 *>(smem + OFF_B2 + ktt_chunk(rowK, d, 8 * th + g)) = w;
-                    }
-                }
-            }
-            fence_proxy_async_smem();
-            __syncthreads();
-            if (slow) {
-                // A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}, j <= i < L, elementwise
-                const float *lg = reinterpret_cast<const float *>(smem + OFF_KT);
-                for (int idx = tid; idx < CH * CH; idx += NT) {
-                    const int i = idx >> 6, j = idx & 63;
-                    float acc = 0.f;
-                    if (j <= i && i < L) {
-                        for (int dd = 0; dd < D; ++dd)
-                            acc = fmaf(bf16f(sQ[i * D + dd]) * bf16f(sK[j * D + dd]),
-                                       ex2(lg[i * D + dd] - lg[j * D + dd]), acc);
-                    }
-                    *reinterpret_cast<float *>(smem + OFF_B2 + a_off(rowA, i, j)) = rna_tf32(acc);
-                }
+            if (!have_prep) {
+                wait_w(bar_tma, ph_tma);
+                build_fast(smem, tmem, L, par);
                 fence_proxy_async_smem();
-                __syncthreads();
+                tc_fence_before();
+                if (!sync_all())
+                    break;
+                prep_fast = guard(state_max());
+                if (prep_fast && tid == kIssuer && has_next)
+                    issue_tma(tok + L);
             }
+            if (!prep_fast) {
+                if (pend) {
+                    if (!wait_all(bar_o, ph_o))
+                        break;
+                    state_pass(smem, tmem, pend_par, ckpt_slot(pend_end), false);
+                    out_epilogue(tmem, out_of(pend_tok), tstride, pend_L, pend_par);
+                    tc_fence_before();
+                    __syncthreads();
+                    tc_fence_after();
+                    pend = false;
+                }
+                if (!exact_segment(tok, L, par, seg_end))
+                    break;
+                if (tid == kIssuer && has_next)
+                    issue_tma(tok + L);
+                pos = seg_end;
+                tok += L;
+                have_prep = false;
+                qk_issued = false;
+                continue;
+            }
+            mk_cur = mk_new;
+            mv_cur = mv_new;
+            if (pend)
+                wait_w(bar_o, ph_o);
+            state_pass(smem, tmem, pend ? pend_par : -1, pend ? ckpt_slot(pend_end) : nullptr, true);
+            tc_fence_before();
+            if (!sync_all())
+                break;
+            const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
             if (tid == kIssuer) {
                 tc_fence_after();
-                if (!slow) {
-                    // Q~ K~^T into D_A
+                if (!qk_issued) {
 #pragma unroll
-                    for (int kk = 0; kk < D / 8; ++kk) {
-                        const uint32_t koff = (kk >> 2) * SLAB + (kk & 3) * 32;
-                        mma_tf32_ss(tmem + TM_A, sdesc_sw128(sb + OFF_QT + koff, 16, 1024),
-                                    sdesc_sw128(sb + OFF_KT + koff, 16, 1024), IDESC_N64, kk > 0);
+                    for (int kk = 0; kk < D / 16; ++kk) {
+                        const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
+                        mma_f16_ss(tmem + TM_A, sdesc_sw128(setb + S_QH + koff, 16, 1024),
+                                   sdesc_sw128(setb + S_KH + koff, 16, 1024), IDF_N64, kk > 0);
                     }
                 }
-                tc_commit(bar_a);     // covers S^T Q~^T too: Q~ is free once it arrives
-                if (has_next)
-                    issue_tma(tok + L);   // the staged inputs have been consumed
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
+                    mma_f16_ts(tmem + (par ? TM_O1 : TM_O0), tmem + TM_SH + kk * 8,
+                               sdesc_sw128(setb + S_QH + koff, 16, 1024), IDF_N64, kk > 0);
+                }
+                tc_commit(bar_a);
             }
-            // output of the previous segment while the tensor core works
-            if (prev_valid)
-                out_epilogue(tok_prev, L_prev, par ^ 1);
+            if (pend)
+                out_epilogue(tmem, out_of(pend_tok), tstride, pend_L, pend_par);
+            pend = false;
+            const bool next_long = has_next && seg_len(seg_end) > kShort;
+            bool next_fast = false;
+            if (next_long) {
+                const int L1 = seg_len(seg_end);
+                wait_w(bar_tma, ph_tma);
+                build_fast(smem, tmem, L1, par ^ 1);
+                fence_proxy_async_smem();
+                tc_fence_before();
+                if (!sync_all())
+                    break;
+                next_fast = guard(state_max() + 64.0f * mk_cur * mv_cur);
+                if (next_fast && tid == kIssuer && seg_end + L1 < end)
+                    issue_tma(tok + L + L1);
+            }
             if (!wait_all(bar_a, ph_a))
                 break;
-            if (!slow && worker && (warp & 3) < 2) {
-                // the causally masked intra-chunk matrix A -> rows rowA.. of [A ; K~^T]
-                const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
-                const int jb = (warp >> 2) * 32;            // this warp's 32 key columns
-                float r[32];
-                tmem_ld32(tmem + lrow + TM_A + jb, r);
-                tmem_wait_ld();
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    float4 w;
-                    float *wv = &w.x;
-#pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        wv[u] = (jb + 4 * c + u <= i) ? rna_tf32(r[4 * c + u]) : 0.f;
-                    const uint32_t o = (jb >> 5) * SLAB_B2 + (rowA + i) * 128 + ((uint32_t)(c ^ (i & 7)) << 4);
-                    *reinterpret_cast<float4 *>(smem + OFF_B2 + o) = w;
-                }
-            }
+            a_build(smem, tmem, par);
             fence_proxy_async_smem();
             tc_fence_before();
-            __syncthreads();
-            if (tid == kIssuer) {
-                // [D_O | S^T] += V^T [A ; K~^T]^T as one N=192 product (V^T from tensor
-                // memory); on the exact path only D_O += V^T A^T here
-                tc_fence_after();
-                const uint32_t vt = tmem + TM_V + 64 * par;
-#pragma unroll
-                for (int kk = 0; kk < CH / 8; ++kk) {
-                    const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32;
-                    if (!slow)
-                        mma_tf32_ts(tmem + (par ? TM_S : TM_O0), vt + kk * 8,
-                                    sdesc_sw128(sb + OFF_B2 + koff, 16, 1024), IDESC_N192, 1);
-                    else
-                        mma_tf32_ts(tmem + tm_o, vt + kk * 8,
-                                    sdesc_sw128(sb + OFF_B2 + koff + rowA * 128, 16, 1024), IDESC_N64, 1);
-                }
-                tc_commit(bar_o);
-            }
-            // next segment's inputs while the tensor core runs the second product
-            if (next_long) {
-                if (!wait_tma())
-                    break;
-                prep(L_next, par ^ 1);
-            }
-            if (!wait_all(bar_o, ph_o))
+            if (!sync_all())
                 break;
-            float *slot = ckpt_slot(seg_end);
-            decay_state(par, slow ? nullptr : slot);
-            if (slow) {
-                tc_fence_before();
-                __syncthreads();
-                if (tid == kIssuer) {
-                    tc_fence_after();
-                    const uint32_t vt = tmem + TM_V + 64 * par;
+            if (tid == kIssuer) {
+                tc_fence_after();
+                const uint32_t vt = tmem + TM_V + 32 * par;
 #pragma unroll
-                    for (int kk = 0; kk < CH / 8; ++kk) {
-                        const uint32_t koff = (kk >> 2) * SLAB_B2 + (kk & 3) * 32 + rowK * 128;
-                        mma_tf32_ts(tmem + TM_S, vt + kk * 8, sdesc_sw128(sb + OFF_B2 + koff, 16, 1024),
-                                    IDESC_N128, 1);
-                    }
-                    tc_commit(bar_s);
-                }
-                if (!wait_all(bar_s, ph_s))
-                    break;
-                if (worker && slot != nullptr) {
+                for (int kk = 0; kk < CH / 16; ++kk)
+                    mma_f16_ts(tmem + (par ? TM_S : TM_O0), vt + kk * 8,
+                               sdesc_sw128(setb + S_B2H + kk * 32, 16, 1024), IDF_N192, 1);
+                tc_commit(bar_o);
+                if (next_fast) {
+                    const uint32_t nsetb = sb + (uint32_t)(par ^ 1) * SET_BYTES;
 #pragma unroll
-                    for (int c0 = 0; c0 < 64; c0 += 32) {
-                        const int d0 = colhalf * 64 + c0;
-                        float r[32];
-                        tmem_ld32(tmem + lrow + TM_S + d0, r);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int x = 0; x < 32; ++x)
-                            slot[(int64_t)(d0 + x) * D + e_own] = r[x];
+                    for (int kk = 0; kk < D / 16; ++kk) {
+                        const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
+                        mma_f16_ss(tmem + TM_A, sdesc_sw128(nsetb + S_QH + koff, 16, 1024),
+                                   sdesc_sw128(nsetb + S_KH + koff, 16, 1024), IDF_N64, kk > 0);
                     }
                 }
             }
-            prev_valid = true;
-            tok_prev = tok;
-            L_prev = L;
+            qk_issued = next_fast;
+            pend = true;
+            pend_par = par;
+            pend_tok = tok;
+            pend_L = L;
+            pend_end = seg_end;
             pos = seg_end;
             tok += L;
             par ^= 1;
-            if (!next_long)
-                break;
+            have_prep = next_long;
+            prep_fast = next_fast;
         }
         if (aborted)
             goto finish;
-        // output of the last pipelined segment
-        out_epilogue(tok_prev, L_prev, par ^ 1);
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
+        if (pend) {
+            if (!wait_all(bar_o, ph_o))
+                goto finish;
+            state_pass(smem, tmem, pend_par, ckpt_slot(pend_end), false);
+            out_epilogue(tmem, out_of(pend_tok), tstride, pend_L, pend_par);
+            tc_fence_before();
+            __syncthreads();
+            tc_fence_after();
+        }
     }
 
     // trailing short segment (its inputs were requested by the previous segment)
@@ -695,8 +1016,8 @@ finish:
     } else if (tid == kIssuer) {
         report(p.d_err, HS_DEVERR_TIMEOUT);
         // let this CTA's own copies and MMAs drain (bounded) before its memory goes away
-        if (tma_inflight)
-            mbar_wait_bounded(bar_tma, ph_tma, kTimeoutNs);
+        if (n_tma > 0)
+            mbar_wait_bounded(bar_tma, (n_tma - 1) & 1, kTimeoutNs);
         tc_commit(bar_s);
         mbar_wait_bounded(bar_s, ph_s, kTimeoutNs);
     }
