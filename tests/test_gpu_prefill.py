@@ -12,7 +12,8 @@ import torch
 
 import oracle
 import paper_2609_15030_gb300 as hs
-from hs_inputs import LONG24, SWEEP, TINY, gen_linear, gen_state
+from hs_inputs import (LONG24, SWEEP, TINY, bf16_bits_to_f32, f32_to_bf16_bits, gen_linear,
+                       gen_state)
 from tests.gpu_helpers import TOL, device, maxnorm_err, run_prefill, to_dev
 
 pytestmark = pytest.mark.gpu
@@ -113,9 +114,9 @@ def test_batch_mixed_positions_from_nonzero_state(kernel, d):
 
 @pytest.mark.parametrize("kernel", KERNELS)
 def test_mixed_gate_strengths_take_both_paths(kernel):
-    """Chunks whose per-dimension decay exceeds 2^-64 (the tensor-core kernel's
-    exact path) interleaved with ordinary chunks; both must match the oracle and
-    keep resume == recompute bitwise."""
+    """Chunks whose per-dimension decay is too strong for the factorised fp16
+    operands (the tensor-core kernel's exact path) interleaved with ordinary
+    chunks; both must match the oracle and keep resume == recompute bitwise."""
     dev = device()
     N, C, nH, d = 448, 64, 4, 128
     inp = gen_linear(12, 0, 1, N, nH, d, d)
@@ -126,6 +127,42 @@ def test_mixed_gate_strengths_take_both_paths(kernel):
     for c in (64, 192, 320):
         o_f, S_f, ck_f = _resume_equals_recompute(inp, N, c, C, dev, kernel)
     _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], "mixed gates")
+
+
+def _scaled(bits, f):
+    return f32_to_bf16_bits(bf16_bits_to_f32(bits) * np.float32(f))
+
+
+@pytest.mark.parametrize("case", ["big_v", "big_qk", "positive_gates", "big_state"])
+def test_fp16_range_guards_take_the_exact_path(case):
+    """Inputs outside the fast path's fp16 range (values, the bound on the intra-chunk
+    scores, growing gates, a large restored state) in some chunks: those chunks take
+    the exact path, the others stay fast; all match the oracle, resume == recompute."""
+    dev = device()
+    N, C, nH, d = 448, 64, 4, 128
+    inp = gen_linear(15, 0, 1, N, nH, d, d)
+    S0 = gen_state(15, 0, 1, nH, d, d)
+    if case == "big_v":
+        inp.v[:, 130:150] = _scaled(inp.v[:, 130:150], 2.0 ** 17)
+    elif case == "big_qk":
+        inp.q[:, 200:260] = _scaled(inp.q[:, 200:260], 64.0)
+        inp.k[:, 200:260] = _scaled(inp.k[:, 200:260], 64.0)
+    elif case == "positive_gates":
+        inp.a[:, 64:128] = 0.02
+    else:
+        S0 = (S0 * 2.0 ** 16).astype(np.float32)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], S0=S0, C_=C)
+    o, S, cks = run_prefill(inp, [0], [N], S0, C, dev, hs.HS_LINATTN_CHUNKED_TC)
+    _check(o, S, cks, ro, rS, rck, [0], [N], case)
+    # resume from the GPU's own checkpoints reproduces the full run bit for bit
+    for c in (64, 192):
+        m = c // C - 1
+        sub = type(inp)(*(x[:, c:N].copy() for x in (inp.q, inp.k, inp.v, inp.a)))
+        o_r, S_r, ck_r = run_prefill(sub, [c], [N - c], cks[0][m][None], C, dev,
+                                     hs.HS_LINATTN_CHUNKED_TC)
+        assert np.array_equal(o_r[0].view(np.uint32), o[0, c:N].view(np.uint32))
+        assert np.array_equal(S_r.view(np.uint32), S.view(np.uint32))
+        assert np.array_equal(ck_r[0].view(np.uint32), cks[0][m + 1:].view(np.uint32))
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
