@@ -24,13 +24,6 @@ template <typename... KArgs, typename... Args>
 inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
                               cudaStream_t stream, Args &&...args)
 {
-    // Every kernel of the library asks for the largest shared-memory carveout, so SMs
-    // keep one L1/shared split across back-to-back launches of different kernels
-    // instead of reconfiguring between them (none of them relies on L1 reuse).
-    cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                         (int)cudaSharedmemCarveoutMaxShared);
-    if (e != cudaSuccess)
-        return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
