@@ -494,10 +494,12 @@ def kv_stress(dev, n_requests=64, staging_pool=4):
             "gbs_aggregate": round(nbytes * len(ts) / sum(ts) / 1e9, 1)}
 
 
-def kv_from_host(dev, n_requests=8, pool=2):
-    """KV-stress requests (48 layers x 256 pages x 64 KiB) restored straight from a
-    pinned host staging pool: the scatter kernel reads host memory over the host link
-    (the paper's CPU cache tier, Section 5.5) and writes the paged cache in HBM."""
+def kv_host(dev, save=False, n_requests=8, pool=2):
+    """KV-stress requests (48 layers x 256 pages x 64 KiB) between the paged cache in HBM
+    and a pinned host staging pool, with no separate copy: restored straight from host
+    memory (the scatter kernel reads it over the host link, the paper's CPU cache tier,
+    Section 5.5), or saved to it (the gather kernel writes it, the save path of
+    Section 3.1)."""
     import torch
     import paper_2609_15030_gb300 as hs
     from hs_inputs import gen_block_table
@@ -505,31 +507,59 @@ def kv_from_host(dev, n_requests=8, pool=2):
     nL, n_pages, P = S.n_full, 4096 // S.page, S.page_bytes
     NB = 4 * n_pages
     cache = torch.empty((nL, NB * P), dtype=torch.uint8, device=dev)
+    cache.view(torch.int32).random_(generator=torch.Generator(device=dev).manual_seed(6))
     cache_ptrs = hs.ptr_array([cache[l] for l in range(nL)], dev)
     host = torch.empty((pool, nL, n_pages * P), dtype=torch.uint8).pin_memory()
     host.view(torch.int32).random_(generator=torch.Generator().manual_seed(5))
     ptrs = [hs.ptr_array([host[i, l] for l in range(nL)], dev) for i in range(pool)]
     bts = [torch.from_numpy(gen_block_table(41, i, n_pages, NB)).to(dev) for i in range(n_requests)]
     stream = torch.cuda.current_stream(dev)
-    hs.hs_restore_kv_pages(ptrs[0], cache_ptrs, nL, bts[0], n_pages, P, NB, None, stream.cuda_stream)
+
+    def move(i):
+        if save:
+            hs.hs_save_kv_pages(cache_ptrs, ptrs[i % pool], nL, bts[i], n_pages, P, NB, None,
+                                stream.cuda_stream)
+        else:
+            hs.hs_restore_kv_pages(ptrs[i % pool], cache_ptrs, nL, bts[i], n_pages, P, NB, None,
+                                   stream.cuda_stream)
+    move(0)
     torch.cuda.synchronize(dev)
     evs = []
     for i in range(n_requests):
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        hs.hs_restore_kv_pages(ptrs[i % pool], cache_ptrs, nL, bts[i], n_pages, P, NB, None,
-                               stream.cuda_stream)
+        move(i)
         e1.record(stream)
         evs.append((e0, e1))
     torch.cuda.synchronize(dev)
     ts = [e0.elapsed_time(e1) * 1e-3 for e0, e1 in evs]
     payload = nL * n_pages * P
-    del cache, host
+    # context: the same bytes as one contiguous copy-engine transfer in the same direction
+    dev_buf = cache[:, :n_pages * P]
+    ce = []
+    for _ in range(3):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        if save:
+            host[0].copy_(dev_buf, non_blocking=True)
+        else:
+            dev_buf.copy_(host[0], non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        ce.append(e0.elapsed_time(e1) * 1e-3)
+    del cache, host, dev_buf
     torch.cuda.empty_cache()
-    return {"bytes_per_request": payload, "median_us": round(statistics.median(ts) * 1e6, 1),
-            "host_read_gbs": round(payload / statistics.median(ts) / 1e9, 1),
-            "source": "pinned host memory (device-accessible), read by the scatter kernel"}
+    out = {"bytes_per_request": payload, "median_us": round(statistics.median(ts) * 1e6, 1),
+           "copy_engine_gbs": round(payload / statistics.median(ce) / 1e9, 1)}
+    if save:
+        out["host_write_gbs"] = round(payload / statistics.median(ts) / 1e9, 1)
+        out["target"] = "pinned host memory (device-accessible), written by the gather kernel"
+    else:
+        out["host_read_gbs"] = round(payload / statistics.median(ts) / 1e9, 1)
+        out["source"] = "pinned host memory (device-accessible), read by the scatter kernel"
+    return out
 
 
 def e2e_run(wl, steps, warmup):
@@ -973,7 +1003,8 @@ def main():
         kv["frac"] = round(kv["gbs_aggregate"] / peak, 4)
         kv["traffic"] = _traffic().get("kv_scatter_kernel@kvstress")
         out["kv_restore"] = kv
-        out["kv_restore_from_host"] = kv_from_host(dev)
+        out["kv_restore_from_host"] = kv_host(dev)
+        out["kv_save_to_host"] = kv_host(dev, save=True)
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
         print(json.dumps(out))

@@ -12,6 +12,8 @@
  *   4. hs_linattn_prefill_from_state   gated linear-attention prefill over the tail [c,N)
  *                                      from that state, emitting state checkpoints.
  *   5. hs_checkpoint_states            snapshot live states into checkpoint slots.
+ *   6. hs_save_kv_pages                gather cache pages by block table into a staging
+ *                                      pool (the save path; device or pinned host memory).
  *
  * Conventions shared by every call
  *   - Every call returns hs_status.  HS_OK means the arguments passed host-side
@@ -125,6 +127,38 @@ hs_status hs_restore_kv_pages(const void *const *staging_layers, void *const *ca
                               int32_t n_layers, const int32_t *block_table, int32_t n_pages,
                               int64_t page_bytes, int64_t num_blocks, int32_t *d_err,
                               cudaStream_t stream);
+
+/*
+ * hs_save_kv_pages -- gather KV pages of the paged cache into a staging pool (save).
+ *
+ * Paper: Section 3.1 (a save must have completed, not merely been submitted,
+ * before dependent state is reused; the final regression delayed every save by
+ * 500 ms and paired each dependent reuse with a wait on the actual save) and
+ * Table 5 (D2H page comparisons, delayed-save wait pairs).
+ *
+ * For every layer l < n_layers and page j < n_pages:
+ *     staging_layers[l] + j*page_bytes  <-  cache_layers[l] + block_table[j]*page_bytes
+ * (page_bytes bytes), the inverse of hs_restore_kv_pages.  The call is
+ * asynchronous: the pages are saved once the stream reaches the copy, so a
+ * caller that will overwrite those cache blocks (or read the staging pool) from
+ * other work must first wait for it, e.g. on a CUDA event recorded on `stream`
+ * after this call.
+ *   cache_layers    device array of n_layers device pointers, each to
+ *                   num_blocks*page_bytes bytes (one layer's paged cache); read only
+ *   staging_layers  device array of n_layers pointers, each to n_pages*page_bytes
+ *                   bytes; device memory, or pinned host memory the device can
+ *                   address (the pages are then written over the host link)
+ *   block_table     device, n_pages int32 block ids, distinct; an id outside
+ *                   [0,num_blocks) sets HS_DEVERR_BLOCK_OOB and that page is skipped
+ *   page_bytes      > 0, multiple of 16
+ * Every pointer in the arrays must be 16-byte aligned (else HS_DEVERR_MISALIGNED
+ * and the layer is skipped).  n_layers == 0 or n_pages == 0 is a no-op.
+ * Errors: HS_ERR_INVALID_ARG, HS_ERR_MISALIGNED (page_bytes), HS_ERR_CUDA.
+ */
+hs_status hs_save_kv_pages(const void *const *cache_layers, void *const *staging_layers,
+                           int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                           int64_t page_bytes, int64_t num_blocks, int32_t *d_err,
+                           cudaStream_t stream);
 
 /*
  * hs_restore_state -- restore recurrent states from checkpoint slots.

@@ -50,6 +50,9 @@ def lib():
             L.oracle_scatter_pages.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
                                                C.c_int32, C.c_int64]
             L.oracle_scatter_pages.restype = None
+            L.oracle_gather_pages.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
+                                              C.c_int32, C.c_int64]
+            L.oracle_gather_pages.restype = None
             L.oracle_copy_slots.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_int64]
             L.oracle_copy_slots.restype = None
             L.oracle_restore_bytes.argtypes = [C.c_int64] * 7
@@ -106,6 +109,13 @@ def scatter_pages(staging_layers, cache_layers, block_table, n_pages: int, page_
     bt = np.ascontiguousarray(block_table, dtype=np.int32)
     lib().oracle_scatter_pages(_ptr_array(staging_layers), _ptr_array(cache_layers),
                                len(cache_layers), bt.ctypes.data, int(n_pages), int(page_bytes))
+
+
+def gather_pages(cache_layers, staging_layers, block_table, n_pages: int, page_bytes: int):
+    """In place on staging_layers (list of uint8 arrays): the save of Section 3.1."""
+    bt = np.ascontiguousarray(block_table, dtype=np.int32)
+    lib().oracle_gather_pages(_ptr_array(cache_layers), _ptr_array(staging_layers),
+                              len(staging_layers), bt.ctypes.data, int(n_pages), int(page_bytes))
 
 
 def copy_slots(src, dst, floats_each: int):

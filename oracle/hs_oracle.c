@@ -19,6 +19,9 @@
  *   - oracle_scatter_pages:    restoring the attention cache entries of
  *                              [0,B) page by page (Section 2.1, Section 5.2),
  *                              as memcpy.
+ *   - oracle_gather_pages:     saving cache pages into a staging pool by block
+ *                              table (the save path of Section 3.1 and the
+ *                              D2H comparisons of Table 5), as memcpy.
  *   - oracle_copy_slots:       restoring / snapshotting the recurrent state
  *                              (Section 1: state updated in place must be
  *                              restored, not recounted), as memcpy.
@@ -111,6 +114,16 @@ void oracle_scatter_pages(const uint8_t *const *staging, uint8_t *const *cache, 
         for (int32_t j = 0; j < n_pages; ++j)
             memcpy(cache[l] + (int64_t)bt[j] * page_bytes,
                    staging[l] + (int64_t)j * page_bytes, (size_t)page_bytes);
+}
+
+/* staging_l[j] <- cache_l[bt[j]] for every layer l and page j < n_pages. */
+void oracle_gather_pages(const uint8_t *const *cache, uint8_t *const *staging, int32_t n_layers,
+                         const int32_t *bt, int32_t n_pages, int64_t page_bytes)
+{
+    for (int32_t l = 0; l < n_layers; ++l)
+        for (int32_t j = 0; j < n_pages; ++j)
+            memcpy(staging[l] + (int64_t)j * page_bytes,
+                   cache[l] + (int64_t)bt[j] * page_bytes, (size_t)page_bytes);
 }
 
 /* dst[i] <- src[i], n slots of floats_each float32 values. */

@@ -126,6 +126,29 @@ hs_status hs_restore_kv_pages(const void *const *staging_layers, void *const *ca
                                              n_pages, page_bytes, num_blocks, d_err, sms, stream));
 }
 
+hs_status hs_save_kv_pages(const void *const *cache_layers, void *const *staging_layers,
+                           int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                           int64_t page_bytes, int64_t num_blocks, int32_t *d_err,
+                           cudaStream_t stream)
+{
+    if (n_layers < 0 || n_pages < 0 || page_bytes <= 0 || num_blocks < 0)
+        return HS_ERR_INVALID_ARG;
+    if (page_bytes % 16 != 0)
+        return HS_ERR_MISALIGNED;
+    if (n_layers == 0 || n_pages == 0)
+        return HS_OK;
+    if (staging_layers == nullptr || cache_layers == nullptr || block_table == nullptr)
+        return HS_ERR_INVALID_ARG;
+    if ((int64_t)n_pages > num_blocks)
+        return HS_ERR_INVALID_ARG;  // a request's pages occupy distinct blocks
+    int sms = 0;
+    hs_status st = sm_count(&sms);
+    if (st != HS_OK)
+        return st;
+    return cuda_status(hs::launch_kv_gather(cache_layers, staging_layers, n_layers, block_table,
+                                            n_pages, page_bytes, num_blocks, d_err, sms, stream));
+}
+
 hs_status hs_restore_state(const float *const *src_slots, float *const *dst_slots, int32_t n,
                            int64_t floats_each, int32_t *d_err, cudaStream_t stream)
 {

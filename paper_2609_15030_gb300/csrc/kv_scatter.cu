@@ -1,6 +1,9 @@
-// Block-table scatter of KV pages from a device staging pool into the paged
-// KV cache (restoring the attention cache entries of the credited prefix,
-// Section 2.1 and Section 5.2 of the paper).
+// Block-table scatter of KV pages from a staging pool into the paged KV cache
+// (restoring the attention cache entries of the credited prefix, Section 2.1
+// and Section 5.2 of the paper), and the inverse gather of cache pages into a
+// staging pool (the save path whose completion Section 3.1 and Table 5 check).
+// Staging may be device memory or pinned host memory read or written over
+// NVLink-C2C.
 //
 // Pure HBM copy: every page is a contiguous run of page_bytes bytes on both
 // sides, so each CTA moves whole pages with 16-byte vector loads and stores.
@@ -28,18 +31,21 @@ __device__ __forceinline__ void st_stream(uint4 *p, const uint4 &v)
     __stcs(p, v);
 }
 
-__global__ void __launch_bounds__(kThreads)
-kv_scatter_kernel(const void *const *staging, void *const *cache, int32_t n_layers,
-                  const int32_t *bt, int32_t n_pages, int64_t page_vecs, int64_t num_blocks,
-                  int32_t *d_err)
+// Page j of every layer moves between staging slot j and cache block bt[j]:
+// cache <- staging when kGather is false, staging <- cache when it is true.
+template <bool kGather>
+__device__ __forceinline__ void kv_pages(const void *const *staging, void *const *cache_w,
+                                         const void *const *cache_r, int32_t n_layers,
+                                         const int32_t *bt, int32_t n_pages, int64_t page_vecs,
+                                         int64_t num_blocks, int32_t *d_err, void *const *staging_w)
 {
     pdl_wait_and_release();
     const int64_t units = (int64_t)n_layers * n_pages;
     for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
         const int32_t l = (int32_t)(u / n_pages);
         const int32_t j = (int32_t)(u - (int64_t)l * n_pages);
-        const uint4 *src = static_cast<const uint4 *>(staging[l]);
-        uint4 *dst = static_cast<uint4 *>(cache[l]);
+        const uint4 *src = static_cast<const uint4 *>(kGather ? cache_r[l] : staging[l]);
+        uint4 *dst = static_cast<uint4 *>(kGather ? staging_w[l] : cache_w[l]);
         const int32_t blk = bt[j];
         if (src == nullptr || dst == nullptr) {
             if (threadIdx.x == 0)
@@ -56,8 +62,8 @@ kv_scatter_kernel(const void *const *staging, void *const *cache, int32_t n_laye
                 report(d_err, HS_DEVERR_BLOCK_OOB);
             continue;
         }
-        src += (int64_t)j * page_vecs;
-        dst += (int64_t)blk * page_vecs;
+        src += (int64_t)(kGather ? blk : j) * page_vecs;
+        dst += (int64_t)(kGather ? j : blk) * page_vecs;
         for (int64_t base = threadIdx.x; base < page_vecs; base += (int64_t)kThreads * kUnroll) {
             uint4 r[kUnroll];
 #pragma unroll
@@ -76,17 +82,48 @@ kv_scatter_kernel(const void *const *staging, void *const *cache, int32_t n_laye
     }
 }
 
+__global__ void __launch_bounds__(kThreads)
+kv_scatter_kernel(const void *const *staging, void *const *cache, int32_t n_layers,
+                  const int32_t *bt, int32_t n_pages, int64_t page_vecs, int64_t num_blocks,
+                  int32_t *d_err)
+{
+    kv_pages<false>(staging, cache, nullptr, n_layers, bt, n_pages, page_vecs, num_blocks, d_err,
+                    nullptr);
+}
+
+__global__ void __launch_bounds__(kThreads)
+kv_gather_kernel(const void *const *cache, void *const *staging, int32_t n_layers,
+                 const int32_t *bt, int32_t n_pages, int64_t page_vecs, int64_t num_blocks,
+                 int32_t *d_err)
+{
+    kv_pages<true>(nullptr, nullptr, cache, n_layers, bt, n_pages, page_vecs, num_blocks, d_err,
+                   staging);
+}
+
+// 8 resident CTAs of 256 threads per SM; at most 4 waves, never more CTAs than units
+int64_t kv_grid(int32_t n_layers, int32_t n_pages, int sm_count)
+{
+    const int64_t units = (int64_t)n_layers * n_pages;
+    const int64_t grid = (int64_t)sm_count * 8 * 4;
+    return grid > units ? units : grid;
+}
+
 }  // namespace
+
+cudaError_t launch_kv_gather(const void *const *cache, void *const *staging, int32_t n_layers,
+                             const int32_t *bt, int32_t n_pages, int64_t page_bytes,
+                             int64_t num_blocks, int32_t *d_err, int sm_count, cudaStream_t s)
+{
+    const int64_t grid = kv_grid(n_layers, n_pages, sm_count);
+    return launch_pdl(kv_gather_kernel, dim3((unsigned)grid), dim3(kThreads), 0, s, cache, staging,
+                      n_layers, bt, n_pages, (int64_t)(page_bytes / 16), num_blocks, d_err);
+}
 
 cudaError_t launch_kv_scatter(const void *const *staging, void *const *cache, int32_t n_layers,
                               const int32_t *bt, int32_t n_pages, int64_t page_bytes,
                               int64_t num_blocks, int32_t *d_err, int sm_count, cudaStream_t s)
 {
-    const int64_t units = (int64_t)n_layers * n_pages;
-    // 8 resident CTAs of 256 threads per SM; at most 4 waves, never more CTAs than units
-    int64_t grid = (int64_t)sm_count * 8 * 4;
-    if (grid > units)
-        grid = units;
+    const int64_t grid = kv_grid(n_layers, n_pages, sm_count);
     return launch_pdl(kv_scatter_kernel, dim3((unsigned)grid), dim3(kThreads), 0, s, staging, cache,
                       n_layers, bt, n_pages, (int64_t)(page_bytes / 16), num_blocks, d_err);
 }

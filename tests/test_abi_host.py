@@ -105,12 +105,13 @@ def test_num_checkpoints_matches_oracle():
 FAKE = 1 << 20        # a 16-byte aligned non-null address that is never dereferenced
 
 
-def test_kv_pages_host_validation():
+@pytest.mark.parametrize("fn", ["hs_restore_kv_pages", "hs_save_kv_pages"])
+def test_kv_pages_host_validation(fn):
     def call(**kw):
         a = dict(staging_layers=FAKE, cache_layers=FAKE, n_layers=1, block_table=FAKE, n_pages=1,
                  page_bytes=64, num_blocks=4, d_err=None, stream=0)
         a.update(kw)
-        hs.hs_restore_kv_pages(**a)
+        getattr(hs, fn)(**a)
     for kw, code in [(dict(n_layers=-1), hs.HS_ERR_INVALID_ARG),
                      (dict(page_bytes=0), hs.HS_ERR_INVALID_ARG),
                      (dict(page_bytes=24), hs.HS_ERR_MISALIGNED),

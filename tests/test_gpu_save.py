@@ -1,0 +1,165 @@
+"""The save path on the GPU: KV pages gathered from the paged cache into a staging
+pool (device or pinned host memory), states snapshotted to host slots, and the
+completion dependency the paper checked with a delayed save (Section 3.1,
+Section 5.3 and Table 5: D2H page comparisons, delayed-save wait pairs).
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2609_15030_gb300 as hs
+from hs_inputs import HYBRID12, gen_block_table
+from tests.gpu_helpers import device
+
+pytestmark = pytest.mark.gpu
+POISON = 0xEE
+
+
+def _cache(dev, L, nb, P, seed):
+    c = torch.empty((L, nb * P), dtype=torch.uint8, device=dev)
+    c.view(torch.int32).random_(generator=torch.Generator(device=dev).manual_seed(seed))
+    return c
+
+
+@pytest.mark.parametrize("where", ["device", "pinned_host"])
+def test_save_pages_match_the_oracle(where):
+    dev = device()
+    L, nb, P, n_pages = 3, 96, HYBRID12.page_bytes, 41
+    cache = _cache(dev, L, nb, P, 5)
+    bt = gen_block_table(21, 0, n_pages, nb)
+    extra = 2                                            # staging pages past n_pages stay poisoned
+    if where == "device":
+        st = torch.full((L, (n_pages + extra) * P), POISON, dtype=torch.uint8, device=dev)
+    else:
+        st = torch.full((L, (n_pages + extra) * P), POISON, dtype=torch.uint8).pin_memory()
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_save_kv_pages(hs.ptr_array([cache[l] for l in range(L)], dev),
+                        hs.ptr_array([st[l] for l in range(L)], dev), L,
+                        torch.from_numpy(bt).to(dev), n_pages, P, nb, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    h_cache = [cache[l].cpu().numpy() for l in range(L)]
+    ref = [np.full((n_pages + extra) * P, POISON, np.uint8) for _ in range(L)]
+    oracle.gather_pages(h_cache, ref, bt, n_pages, P)
+    got = st.cpu().numpy()
+    for l in range(L):
+        assert np.array_equal(got[l], ref[l]), l
+        assert got[l][:n_pages * P].any()                 # the compared bytes are not all zero
+
+
+def test_save_then_restore_round_trip():
+    """Pages saved from one cache and restored into a poisoned one at the same blocks
+    come back bit for bit; other blocks stay poisoned (Table 5's two directions)."""
+    dev = device()
+    L, nb, P, n_pages = 3, 80, HYBRID12.page_bytes, 37
+    a = _cache(dev, L, nb, P, 9)
+    bt = torch.from_numpy(gen_block_table(22, 0, n_pages, nb)).to(dev)
+    st = torch.empty((L, n_pages * P), dtype=torch.uint8).pin_memory()
+    b = torch.full((L, nb * P), POISON, dtype=torch.uint8, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    ap = hs.ptr_array([a[l] for l in range(L)], dev)
+    sp = hs.ptr_array([st[l] for l in range(L)], dev)
+    bp = hs.ptr_array([b[l] for l in range(L)], dev)
+    hs.hs_save_kv_pages(ap, sp, L, bt, n_pages, P, nb, err)
+    hs.hs_restore_kv_pages(sp, bp, L, bt, n_pages, P, nb, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    av, bv = a.view(L, nb, P), b.view(L, nb, P)
+    idx = bt.long()
+    assert torch.equal(bv[:, idx], av[:, idx])
+    mask = torch.ones(nb, dtype=torch.bool, device=dev)
+    mask[idx] = False
+    assert bool((bv[:, mask] == POISON).all())
+
+
+def test_save_out_of_range_block_reports_and_skips():
+    dev = device()
+    P, nb = 4096, 6
+    cache = _cache(dev, 1, nb, P, 3)
+    st = torch.full((3 * P,), POISON, dtype=torch.uint8, device=dev)
+    bt = torch.tensor([4, 6, 1], dtype=torch.int32, device=dev)          # 6 is out of range
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_save_kv_pages(hs.ptr_array([cache], dev), hs.ptr_array([st], dev), 1, bt, 3, P, nb, err)
+    torch.cuda.synchronize()
+    assert err.item() == hs.HS_DEVERR_BLOCK_OOB
+    c = cache.cpu().numpy().reshape(nb, P)
+    s = st.cpu().numpy().reshape(3, P)
+    assert np.array_equal(s[0], c[4]) and np.array_equal(s[2], c[1])
+    assert (s[1] == POISON).all()
+
+
+def test_checkpoint_states_to_pinned_host_slots():
+    """States snapshotted straight into pinned host slots (the checkpoint half of the
+    save), bit for bit."""
+    dev = device()
+    n, fe = 4, HYBRID12.n_heads * HYBRID12.d * HYBRID12.d
+    src = [torch.randn(fe, device=dev) for _ in range(n)]
+    dst = [torch.full((fe,), -3.0).pin_memory() for _ in range(n)]
+    hs.hs_checkpoint_states(hs.ptr_array(src, dev), hs.ptr_array(dst, dev), n, fe)
+    torch.cuda.synchronize()
+    for s, d in zip(src, dst):
+        assert torch.equal(s.cpu().view(torch.int32), d.view(torch.int32))
+
+
+def _driver():
+    for name in ("libcuda.so.1", "libcuda.so"):
+        try:
+            return ctypes.CDLL(name)
+        except OSError:
+            continue
+    pytest.skip("CUDA driver library not found")
+
+
+def test_delayed_saves_complete_before_dependent_reuse():
+    """Each save is followed, on its stream, by a host step that sleeps 500 ms before
+    the save counts as complete (the paper's injected delay); the reuse stream waits on
+    the completion event of every save before it overwrites those cache blocks.  The
+    host staging must hold the pre-overwrite pages, the cache the new ones, and every
+    overwrite must start after its delayed save ended (Section 3.1, Table 5)."""
+    dev = device()
+    drv = _driver()
+    # the injected delay: the driver calls libc usleep(500000) on its own thread (the
+    # host-function argument is the microsecond count), so no Python runs there
+    usleep = ctypes.cast(ctypes.CDLL("libc.so.6").usleep, ctypes.c_void_p)
+    drv.cuLaunchHostFunc.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
+    drv.cuLaunchHostFunc.restype = ctypes.c_int
+
+    L, nb, P, n_saves, m = 3, 64, HYBRID12.page_bytes, 3, 8
+    cache = _cache(dev, L, nb, P, 31)
+    before = cache.clone()
+    new_pages = _cache(dev, L, m, P, 32)                 # what each reuse writes into its blocks
+    s_save, s_reuse = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    cp = hs.ptr_array([cache[l] for l in range(L)], dev)
+    npp = hs.ptr_array([new_pages[l] for l in range(L)], dev)
+    # disjoint block sets, one per save; every buffer and pointer array stays referenced
+    # until the streams drain
+    perm = gen_block_table(40, 0, n_saves * m, nb)
+    bts = [torch.from_numpy(perm[i * m:(i + 1) * m].copy()).to(dev) for i in range(n_saves)]
+    stagings = [torch.full((L, m * P), POISON, dtype=torch.uint8).pin_memory() for _ in range(n_saves)]
+    sps = [hs.ptr_array([st[l] for l in range(L)], dev) for st in stagings]
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(n_saves)]
+    torch.cuda.synchronize()
+    for i in range(n_saves):
+        e_save0, e_saved, e_reuse = events[i]
+        e_save0.record(s_save)
+        hs.hs_save_kv_pages(cp, sps[i], L, bts[i], m, P, nb, err, stream=s_save)
+        assert drv.cuLaunchHostFunc(ctypes.c_void_p(s_save.cuda_stream), usleep,
+                                    ctypes.c_void_p(500000)) == 0
+        e_saved.record(s_save)
+        s_reuse.wait_event(e_saved)                      # the actual completion, not submission
+        e_reuse.record(s_reuse)
+        hs.hs_restore_kv_pages(npp, cp, L, bts[i], m, P, nb, err, stream=s_reuse)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    cv, bv, nv = cache.view(L, nb, P), before.view(L, nb, P), new_pages.view(L, m, P)
+    for i in range(n_saves):
+        idx = bts[i].long()
+        # saved bytes are the pages as they were before the dependent overwrite
+        assert torch.equal(stagings[i].view(L, m, P), bv[:, idx].cpu())
+        # the overwrite happened, and only after the delayed save had completed
+        assert torch.equal(cv[:, idx], nv)
+        assert events[i][0].elapsed_time(events[i][2]) >= 500.0

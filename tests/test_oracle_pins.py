@@ -285,6 +285,27 @@ def test_scatter_pages_and_untouched_bytes():
             assert (cache[l][b * P:(b + 1) * P] == 0xFF).all()
 
 
+def test_gather_pages_reads_each_block_and_inverts_the_scatter():
+    """The save path (Section 3.1): page j of the staging pool is cache block bt[j].
+    Cache bytes encode (layer, block, offset), so a page landing from the wrong block
+    or layer, or shifted, is caught; scatter after gather restores the cache blocks."""
+    P, nb, L = 48, 10, 3
+    cache = [np.array([(l * 37 + b * 5 + (i % 7)) % 251 for b in range(nb) for i in range(P)],
+                      np.uint8) for l in range(L)]
+    bt = np.array([9, 0, 4, 6], np.int32)
+    staging = [np.zeros(len(bt) * P, np.uint8) for _ in range(L)]
+    oracle.gather_pages(cache, staging, bt, len(bt), P)
+    for l in range(L):
+        for j, b in enumerate(bt):
+            want = np.array([(l * 37 + int(b) * 5 + (i % 7)) % 251 for i in range(P)], np.uint8)
+            assert np.array_equal(staging[l][j * P:(j + 1) * P], want)
+    back = [np.full(nb * P, 0xFF, np.uint8) for _ in range(L)]
+    oracle.scatter_pages(staging, back, bt, len(bt), P)
+    for l in range(L):
+        for b in bt:
+            assert np.array_equal(back[l][b * P:(b + 1) * P], cache[l][b * P:(b + 1) * P])
+
+
 def test_bf16_rounding_is_round_to_nearest_even():
     # 1 + 2^-8 is halfway between bf16 neighbours 1 and 1 + 2^-7: ties go to even (1.0)
     x = np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -2.5, 0.0], np.float32)
