@@ -562,6 +562,50 @@ def kv_host(dev, save=False, n_requests=8, pool=2):
     return out
 
 
+def kv_rank_slices(dev, n_requests=16):
+    """One tensor-parallel rank's restore of FP8 KV pages (Table 1: TP=4, FP8 KV): 48
+    layers x 256 pages of 16 tokens x 8 KV heads x 128 (one byte each, 32 KiB pages);
+    the rank moves its 2 heads of every page row (8 KiB per page) from a device staging
+    pool into a paged cache."""
+    import torch
+    import paper_2609_15030_gb300 as hs
+    from hs_inputs import gen_block_table
+    nL, n_pages, tokens, kvh, hd, TP = 48, 256, 16, 8, 128, 4
+    rows, row_bytes = 2 * tokens, kvh * hd
+    P, cb = rows * row_bytes, row_bytes // TP
+    NB = 4 * n_pages
+    cache = torch.zeros((nL, NB * P), dtype=torch.uint8, device=dev)
+    stg = torch.empty((2, nL, n_pages * rows * cb), dtype=torch.uint8, device=dev)
+    stg.view(torch.int32).random_(generator=torch.Generator(device=dev).manual_seed(8))
+    cache_ptrs = hs.ptr_array([cache[l] for l in range(nL)], dev)
+    sps = [hs.ptr_array([stg[i, l] for l in range(nL)], dev) for i in range(2)]
+    bts = [torch.from_numpy(gen_block_table(44, i, n_pages, NB)).to(dev) for i in range(n_requests)]
+    stream = torch.cuda.current_stream(dev)
+
+    def move(i):
+        hs.hs_restore_kv_page_slices(sps[i % 2], cache_ptrs, nL, bts[i], n_pages, P, rows, 0, cb,
+                                     NB, None, stream.cuda_stream)
+    move(0)
+    torch.cuda.synchronize(dev)
+    evs = []
+    for i in range(n_requests):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        move(i)
+        e1.record(stream)
+        evs.append((e0, e1))
+    torch.cuda.synchronize(dev)
+    ts = [e0.elapsed_time(e1) * 1e-3 for e0, e1 in evs]
+    moved = 2 * nL * n_pages * rows * cb            # read + write
+    del cache, stg
+    torch.cuda.empty_cache()
+    t = statistics.median(ts)
+    return {"bytes_per_request": moved, "median_us": round(t * 1e6, 1),
+            "gbs": round(moved / t / 1e9, 1), "slice": f"{cb} of {row_bytes} bytes per row, "
+            f"{rows} rows per {P}-byte page"}
+
+
 def e2e_run(wl, steps, warmup):
     """Same step with every request's inputs in pinned host memory (KV staging
     pages, checkpoint state, q/k/v/log-gates) copied to the device inside the
@@ -1005,6 +1049,9 @@ def main():
         out["kv_restore"] = kv
         out["kv_restore_from_host"] = kv_host(dev)
         out["kv_save_to_host"] = kv_host(dev, save=True)
+        sl = kv_rank_slices(dev)
+        sl["frac"] = round(sl["gbs"] / peak, 4)
+        out["kv_restore_rank_slice_fp8"] = sl
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
         print(json.dumps(out))

@@ -14,6 +14,8 @@
  *   5. hs_checkpoint_states            snapshot live states into checkpoint slots.
  *   6. hs_save_kv_pages                gather cache pages by block table into a staging
  *                                      pool (the save path; device or pinned host memory).
+ *   hs_restore_kv_page_slices / hs_save_kv_page_slices: the same for one tensor-parallel
+ *                                      rank's heads of every page.
  *
  * Conventions shared by every call
  *   - Every call returns hs_status.  HS_OK means the arguments passed host-side
@@ -159,6 +161,42 @@ hs_status hs_save_kv_pages(const void *const *cache_layers, void *const *staging
                            int32_t n_layers, const int32_t *block_table, int32_t n_pages,
                            int64_t page_bytes, int64_t num_blocks, int32_t *d_err,
                            cudaStream_t stream);
+
+/*
+ * hs_restore_kv_page_slices / hs_save_kv_page_slices -- one tensor-parallel rank's
+ * slice of every KV page (restore: staging -> cache; save: cache -> staging).
+ *
+ * Paper: Table 1 (four-way tensor parallelism, FP8 KV setting) and Section 5.2
+ * (restored bytes are counted per rank: each rank moves the pages of its own
+ * heads).
+ *
+ * A page of page_bytes bytes is `rows` rows of row_bytes = page_bytes / rows bytes
+ * (for the cache layout [2][page][kv head][head_dim]: rows = 2*page tokens, a row
+ * = every KV head of one token); a rank owns bytes [col_off, col_off + col_bytes)
+ * of every row (its KV heads).  The staging page holds the rank's rows back to
+ * back, rows*col_bytes bytes, page after page.  For every layer l and page j:
+ *     for r < rows:  cache_l[block_table[j]] + r*row_bytes + col_off   (col_bytes bytes)
+ *                    <->  staging_l + (j*rows + r)*col_bytes
+ * Bytes outside the slices are not written.  The element type is irrelevant (FP8
+ * and BF16 pages are the same bytes to move).  rows = 1, col_off = 0,
+ * col_bytes = page_bytes is hs_restore_kv_pages / hs_save_kv_pages.
+ *   staging_layers, cache_layers, block_table, num_blocks, d_err: as for
+ *                   hs_restore_kv_pages (staging may be pinned host memory)
+ *   rows            >= 1, divides page_bytes
+ *   col_off, col_bytes  col_off >= 0, col_bytes > 0, col_off + col_bytes <= row_bytes
+ * Errors: HS_ERR_INVALID_ARG (sizes, slice outside the row), HS_ERR_MISALIGNED
+ * (page_bytes, row_bytes, col_off or col_bytes not a multiple of 16), HS_ERR_CUDA.
+ */
+hs_status hs_restore_kv_page_slices(const void *const *staging_layers, void *const *cache_layers,
+                                    int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                                    int64_t page_bytes, int32_t rows, int64_t col_off,
+                                    int64_t col_bytes, int64_t num_blocks, int32_t *d_err,
+                                    cudaStream_t stream);
+hs_status hs_save_kv_page_slices(const void *const *cache_layers, void *const *staging_layers,
+                                 int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                                 int64_t page_bytes, int32_t rows, int64_t col_off,
+                                 int64_t col_bytes, int64_t num_blocks, int32_t *d_err,
+                                 cudaStream_t stream);
 
 /*
  * hs_restore_state -- restore recurrent states from checkpoint slots.

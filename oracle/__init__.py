@@ -53,6 +53,9 @@ def lib():
             L.oracle_gather_pages.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
                                               C.c_int32, C.c_int64]
             L.oracle_gather_pages.restype = None
+            L.oracle_slices.argtypes = [C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
+                                        C.c_int32, C.c_int64, C.c_int32, C.c_int64, C.c_int64]
+            L.oracle_slices.restype = None
             L.oracle_copy_slots.argtypes = [C.c_void_p, C.c_void_p, C.c_int32, C.c_int64]
             L.oracle_copy_slots.restype = None
             L.oracle_restore_bytes.argtypes = [C.c_int64] * 7
@@ -116,6 +119,24 @@ def gather_pages(cache_layers, staging_layers, block_table, n_pages: int, page_b
     bt = np.ascontiguousarray(block_table, dtype=np.int32)
     lib().oracle_gather_pages(_ptr_array(cache_layers), _ptr_array(staging_layers),
                               len(staging_layers), bt.ctypes.data, int(n_pages), int(page_bytes))
+
+
+def scatter_slices(staging_layers, cache_layers, block_table, n_pages: int, page_bytes: int,
+                   rows: int, col_off: int, col_bytes: int):
+    """One rank's slice of every page row, staging -> cache, in place on cache_layers."""
+    bt = np.ascontiguousarray(block_table, dtype=np.int32)
+    lib().oracle_slices(0, _ptr_array(staging_layers), _ptr_array(cache_layers), len(cache_layers),
+                        bt.ctypes.data, int(n_pages), int(page_bytes), int(rows), int(col_off),
+                        int(col_bytes))
+
+
+def gather_slices(cache_layers, staging_layers, block_table, n_pages: int, page_bytes: int,
+                  rows: int, col_off: int, col_bytes: int):
+    """One rank's slice of every page row, cache -> staging, in place on staging_layers."""
+    bt = np.ascontiguousarray(block_table, dtype=np.int32)
+    lib().oracle_slices(1, _ptr_array(staging_layers), _ptr_array(cache_layers),
+                        len(staging_layers), bt.ctypes.data, int(n_pages), int(page_bytes),
+                        int(rows), int(col_off), int(col_bytes))
 
 
 def copy_slots(src, dst, floats_each: int):

@@ -22,6 +22,9 @@
  *   - oracle_gather_pages:     saving cache pages into a staging pool by block
  *                              table (the save path of Section 3.1 and the
  *                              D2H comparisons of Table 5), as memcpy.
+ *   - oracle_scatter_slices / oracle_gather_slices: the same for one tensor-
+ *                              parallel rank's bytes of every page row (Table 1:
+ *                              TP=4; Section 5.2: per-rank transfers), as memcpy.
  *   - oracle_copy_slots:       restoring / snapshotting the recurrent state
  *                              (Section 1: state updated in place must be
  *                              restored, not recounted), as memcpy.
@@ -124,6 +127,27 @@ void oracle_gather_pages(const uint8_t *const *cache, uint8_t *const *staging, i
         for (int32_t j = 0; j < n_pages; ++j)
             memcpy(staging[l] + (int64_t)j * page_bytes,
                    cache[l] + (int64_t)bt[j] * page_bytes, (size_t)page_bytes);
+}
+
+/* For every layer l, page j, row r < rows of row_bytes = page_bytes/rows:
+ * bytes [col_off, col_off+col_bytes) of row r of cache_l[bt[j]] and the packed
+ * staging row staging_l[(j*rows + r)*col_bytes ...]; gather != 0 copies cache to
+ * staging, else staging to cache. */
+void oracle_slices(int32_t gather, uint8_t *const *staging, uint8_t *const *cache, int32_t n_layers,
+                   const int32_t *bt, int32_t n_pages, int64_t page_bytes, int32_t rows,
+                   int64_t col_off, int64_t col_bytes)
+{
+    const int64_t row_bytes = page_bytes / rows;
+    for (int32_t l = 0; l < n_layers; ++l)
+        for (int32_t j = 0; j < n_pages; ++j)
+            for (int32_t r = 0; r < rows; ++r) {
+                uint8_t *c = cache[l] + (int64_t)bt[j] * page_bytes + r * row_bytes + col_off;
+                uint8_t *s = staging[l] + ((int64_t)j * rows + r) * col_bytes;
+                if (gather)
+                    memcpy(s, c, (size_t)col_bytes);
+                else
+                    memcpy(c, s, (size_t)col_bytes);
+            }
 }
 
 /* dst[i] <- src[i], n slots of floats_each float32 values. */

@@ -149,6 +149,56 @@ hs_status hs_save_kv_pages(const void *const *cache_layers, void *const *staging
                                             n_pages, page_bytes, num_blocks, d_err, sms, stream));
 }
 
+static hs_status kv_slices(bool gather, const void *const *from, void *const *to, int32_t n_layers,
+                           const int32_t *block_table, int32_t n_pages, int64_t page_bytes,
+                           int32_t rows, int64_t col_off, int64_t col_bytes, int64_t num_blocks,
+                           int32_t *d_err, cudaStream_t stream)
+{
+    if (n_layers < 0 || n_pages < 0 || page_bytes <= 0 || num_blocks < 0 || rows <= 0 ||
+        col_off < 0 || col_bytes <= 0)
+        return HS_ERR_INVALID_ARG;
+    if (page_bytes % rows != 0 || col_off + col_bytes > page_bytes / rows)
+        return HS_ERR_INVALID_ARG;
+    if (page_bytes % 16 != 0 || (page_bytes / rows) % 16 != 0 || col_off % 16 != 0 ||
+        col_bytes % 16 != 0)
+        return HS_ERR_MISALIGNED;
+    if ((int64_t)rows * (col_bytes / 16) > INT32_MAX)
+        return HS_ERR_UNSUPPORTED;   // one page slice is at most 2^31 16-byte vectors
+    if (n_layers == 0 || n_pages == 0)
+        return HS_OK;
+    if (from == nullptr || to == nullptr || block_table == nullptr)
+        return HS_ERR_INVALID_ARG;
+    if ((int64_t)n_pages > num_blocks)
+        return HS_ERR_INVALID_ARG;  // a request's pages occupy distinct blocks
+    int sms = 0;
+    hs_status st = sm_count(&sms);
+    if (st != HS_OK)
+        return st;
+    return cuda_status(hs::launch_kv_slices(gather, from, to, n_layers, block_table, n_pages,
+                                            page_bytes, rows, col_off, col_bytes, num_blocks, d_err,
+                                            sms, stream));
+}
+
+hs_status hs_restore_kv_page_slices(const void *const *staging_layers, void *const *cache_layers,
+                                    int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                                    int64_t page_bytes, int32_t rows, int64_t col_off,
+                                    int64_t col_bytes, int64_t num_blocks, int32_t *d_err,
+                                    cudaStream_t stream)
+{
+    return kv_slices(false, staging_layers, cache_layers, n_layers, block_table, n_pages,
+                     page_bytes, rows, col_off, col_bytes, num_blocks, d_err, stream);
+}
+
+hs_status hs_save_kv_page_slices(const void *const *cache_layers, void *const *staging_layers,
+                                 int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                                 int64_t page_bytes, int32_t rows, int64_t col_off,
+                                 int64_t col_bytes, int64_t num_blocks, int32_t *d_err,
+                                 cudaStream_t stream)
+{
+    return kv_slices(true, cache_layers, staging_layers, n_layers, block_table, n_pages,
+                     page_bytes, rows, col_off, col_bytes, num_blocks, d_err, stream);
+}
+
 hs_status hs_restore_state(const float *const *src_slots, float *const *dst_slots, int32_t n,
                            int64_t floats_each, int32_t *d_err, cudaStream_t stream)
 {

@@ -71,6 +71,10 @@ cudaError_t launch_kv_scatter(const void *const *staging, void *const *cache, in
 cudaError_t launch_kv_gather(const void *const *cache, void *const *staging, int32_t n_layers,
                              const int32_t *bt, int32_t n_pages, int64_t page_bytes,
                              int64_t num_blocks, int32_t *d_err, int sm_count, cudaStream_t s);
+cudaError_t launch_kv_slices(bool gather, const void *const *from, void *const *to, int32_t n_layers,
+                             const int32_t *bt, int32_t n_pages, int64_t page_bytes, int32_t rows,
+                             int64_t col_off, int64_t col_bytes, int64_t num_blocks, int32_t *d_err,
+                             int sm_count, cudaStream_t s);
 cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t n,
                              int64_t floats_each, int32_t *d_err, int sm_count, cudaStream_t s);
 cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);

@@ -125,6 +125,32 @@ def test_kv_pages_host_validation(fn):
     call(n_pages=0)
 
 
+@pytest.mark.parametrize("fn", ["hs_restore_kv_page_slices", "hs_save_kv_page_slices"])
+def test_kv_page_slices_host_validation(fn):
+    def call(**kw):
+        a = dict(staging_layers=FAKE, cache_layers=FAKE, n_layers=1, block_table=FAKE, n_pages=1,
+                 page_bytes=1024, rows=4, col_off=64, col_bytes=64, num_blocks=4, d_err=None,
+                 stream=0)
+        a.update(kw)
+        if fn == "hs_save_kv_page_slices":
+            a["cache_layers"], a["staging_layers"] = a.pop("cache_layers"), a.pop("staging_layers")
+        getattr(hs, fn)(**a)
+    for kw, code in [(dict(rows=0), hs.HS_ERR_INVALID_ARG),
+                     (dict(rows=3), hs.HS_ERR_INVALID_ARG),            # 3 does not divide 1024
+                     (dict(col_off=224, col_bytes=64), hs.HS_ERR_INVALID_ARG),   # past the row
+                     (dict(col_bytes=0), hs.HS_ERR_INVALID_ARG),
+                     (dict(col_off=8), hs.HS_ERR_MISALIGNED),
+                     (dict(col_bytes=40), hs.HS_ERR_MISALIGNED),
+                     (dict(page_bytes=1032, rows=2), hs.HS_ERR_MISALIGNED),
+                     (dict(block_table=None), hs.HS_ERR_INVALID_ARG),
+                     (dict(n_pages=5, num_blocks=4), hs.HS_ERR_INVALID_ARG)]:
+        with pytest.raises(hs.HsError) as e:
+            call(**kw)
+        assert e.value.status == code, kw
+    call(n_layers=0)
+    call(n_pages=0)
+
+
 def test_state_copy_host_validation():
     for fn in (hs.hs_restore_state, hs.hs_checkpoint_states):
         with pytest.raises(hs.HsError):

@@ -163,3 +163,81 @@ def test_delayed_saves_complete_before_dependent_reuse():
         # the overwrite happened, and only after the delayed save had completed
         assert torch.equal(cv[:, idx], nv)
         assert events[i][0].elapsed_time(events[i][2]) >= 500.0
+
+
+@pytest.mark.parametrize("where", ["device", "pinned_host"])
+def test_fp8_rank_slices_restore_and_save(where):
+    """FP8 KV pages (16 tokens x 8 KV heads x 128, one byte per element) moved as four
+    tensor-parallel ranks' head slices (Table 1: TP=4, FP8 KV; Section 5.2: per-rank
+    transfers): the four restores reassemble the oracle's full-page scatter bit for bit
+    with untouched blocks poisoned, and each rank's save is its oracle gather."""
+    dev = device()
+    tokens, kvh, hd, TP = 16, 8, 128, 4
+    rows, row_bytes = 2 * tokens, kvh * hd
+    P = rows * row_bytes
+    cb = row_bytes // TP
+    L, nb, n_pages = 3, 72, 29
+    rng = np.random.default_rng(17)
+    full = [rng.integers(0, 256, size=n_pages * P, dtype=np.uint8) for _ in range(L)]
+    bt = gen_block_table(23, 0, n_pages, nb)
+    d_bt = torch.from_numpy(bt).to(dev)
+    cache = torch.full((L, nb * P), POISON, dtype=torch.uint8, device=dev)
+    cp = hs.ptr_array([cache[l] for l in range(L)], dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    keep = []
+    for r in range(TP):
+        st = np.stack([f.reshape(n_pages, rows, row_bytes)[:, :, r * cb:(r + 1) * cb].reshape(-1)
+                       for f in full])
+        t = torch.from_numpy(st)
+        t = t.to(dev) if where == "device" else t.pin_memory()
+        keep.append(t)
+        hs.hs_restore_kv_page_slices(hs.ptr_array([t[l] for l in range(L)], dev), cp, L, d_bt,
+                                     n_pages, P, rows, r * cb, cb, nb, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    want = [np.full(nb * P, POISON, np.uint8) for _ in range(L)]
+    oracle.scatter_pages(full, want, bt, n_pages, P)
+    got = cache.cpu().numpy()
+    for l in range(L):
+        assert np.array_equal(got[l], want[l]), l
+    # each rank saves its slice back
+    for r in range(TP):
+        out = torch.full((L, n_pages * rows * cb), POISON, dtype=torch.uint8)
+        out = out.to(dev) if where == "device" else out.pin_memory()
+        hs.hs_save_kv_page_slices(cp, hs.ptr_array([out[l] for l in range(L)], dev), L, d_bt,
+                                  n_pages, P, rows, r * cb, cb, nb, err)
+        torch.cuda.synchronize()
+        assert err.item() == 0
+        ref = [np.zeros(n_pages * rows * cb, np.uint8) for _ in range(L)]
+        oracle.gather_slices([got[l] for l in range(L)], ref, bt, n_pages, P, rows, r * cb, cb)
+        o = out.cpu().numpy()
+        for l in range(L):
+            assert np.array_equal(o[l], ref[l]), (r, l)
+
+
+def test_rank_slices_with_a_row_split_that_does_not_divide_the_block():
+    """Slices of 3 x 16 bytes (a 3-head rank of 12 one-byte-per-dim heads... any split):
+    the general per-vector path; restore then save round-trips bit for bit."""
+    dev = device()
+    L, nb, n_pages, rows, row_bytes, off, cb = 2, 20, 9, 24, 192, 64, 48
+    P = rows * row_bytes
+    rng = np.random.default_rng(19)
+    st = torch.from_numpy(rng.integers(0, 256, size=(L, n_pages * rows * cb), dtype=np.uint8)).to(dev)
+    cache = torch.full((L, nb * P), POISON, dtype=torch.uint8, device=dev)
+    bt = torch.from_numpy(gen_block_table(24, 0, n_pages, nb)).to(dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    cp = hs.ptr_array([cache[l] for l in range(L)], dev)
+    hs.hs_restore_kv_page_slices(hs.ptr_array([st[l] for l in range(L)], dev), cp, L, bt, n_pages,
+                                 P, rows, off, cb, nb, err)
+    back = torch.zeros_like(st)
+    hs.hs_save_kv_page_slices(cp, hs.ptr_array([back[l] for l in range(L)], dev), L, bt, n_pages,
+                              P, rows, off, cb, nb, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    assert torch.equal(back, st)
+    want = [np.full(nb * P, POISON, np.uint8) for _ in range(L)]
+    oracle.scatter_slices([st[l].cpu().numpy() for l in range(L)], want, bt.cpu().numpy(), n_pages,
+                          P, rows, off, cb)
+    got = cache.cpu().numpy()
+    for l in range(L):
+        assert np.array_equal(got[l], want[l])

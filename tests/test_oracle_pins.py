@@ -306,6 +306,35 @@ def test_gather_pages_reads_each_block_and_inverts_the_scatter():
             assert np.array_equal(back[l][b * P:(b + 1) * P], cache[l][b * P:(b + 1) * P])
 
 
+def test_rank_slices_reassemble_the_full_page_transfer():
+    """Four tensor-parallel ranks each move their bytes of every page row (Table 1: TP=4,
+    FP8 pages; Section 5.2: per-rank transfers).  Restoring every rank's slice equals the
+    full-page scatter; each rank's gathered slice is its columns of the full-page gather;
+    each rank moves a quarter of the bytes."""
+    rng = np.random.default_rng(13)
+    tokens, heads, hd, TP, L, nb = 4, 8, 16, 4, 2, 7
+    rows, row_bytes = 2 * tokens, heads * hd              # FP8: one byte per element
+    P = rows * row_bytes
+    cb = row_bytes // TP
+    bt = np.array([5, 1, 3], np.int32)
+    full = [rng.integers(0, 256, size=len(bt) * P, dtype=np.uint8) for _ in range(L)]
+    want = [np.full(nb * P, 0xAB, np.uint8) for _ in range(L)]
+    oracle.scatter_pages(full, want, bt, len(bt), P)
+    got = [np.full(nb * P, 0xAB, np.uint8) for _ in range(L)]
+    for r in range(TP):
+        # rank r's staging: its bytes of every row, rows back to back
+        st = [f.reshape(len(bt), rows, row_bytes)[:, :, r * cb:(r + 1) * cb].copy().reshape(-1)
+              for f in full]
+        assert sum(x.size for x in st) * TP == sum(x.size for x in full)
+        oracle.scatter_slices(st, got, bt, len(bt), P, rows, r * cb, cb)
+        back = [np.zeros_like(x) for x in st]
+        oracle.gather_slices(want, back, bt, len(bt), P, rows, r * cb, cb)
+        for a, b in zip(back, st):
+            assert np.array_equal(a, b)
+    for a, b in zip(got, want):
+        assert np.array_equal(a, b)
+
+
 def test_bf16_rounding_is_round_to_nearest_even():
     # 1 + 2^-8 is halfway between bf16 neighbours 1 and 1 + 2^-7: ties go to even (1.0)
     x = np.array([1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, -2.5, 0.0], np.float32)
