@@ -63,7 +63,7 @@ typedef enum hs_status {
 #define HS_DEVERR_TIMEOUT 4       /* a bounded wait inside a kernel ran out */
 
 /* Largest batch accepted by hs_linattn_prefill_from_state. */
-#define HS_MAX_BATCH 512
+#define HS_MAX_BATCH 384
 /* Chunk length of the prefill; checkpoint intervals are multiples of it. */
 #define HS_CHUNK 64
 /* Segments (the part of a call inside one chunk) of at most this many tokens are
@@ -294,8 +294,10 @@ typedef struct hs_linattn_shape {
  *   d_err      optional device int32 (see conventions)
  * All of q, k, v, log_g, o, state must be 16-byte aligned.  q/k/v/log_g are only
  * read; o, state and the slots must not overlap the inputs or each other.
+ * Token rows are 32-bit: b*max_tokens + n_tokens[b] must stay below 2^31.
  * Errors: HS_ERR_INVALID_ARG, HS_ERR_MISALIGNED, HS_ERR_UNSUPPORTED (d_k/d_v,
- * ckpt_interval not a multiple of HS_CHUNK, batch > HS_MAX_BATCH), HS_ERR_CUDA.
+ * ckpt_interval not a multiple of HS_CHUNK, batch > HS_MAX_BATCH, rows beyond
+ * 2^31), HS_ERR_CUDA.
  */
 hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint16_t *q,
                                         const uint16_t *k, const uint16_t *v, const float *log_g,
@@ -303,6 +305,29 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
                                         const int32_t *n_tokens, int32_t ckpt_interval,
                                         float *const *ckpt_slots, int32_t *d_err,
                                         cudaStream_t stream);
+
+/*
+ * hs_linattn_prefill_packed -- hs_linattn_prefill_from_state over a packed
+ * (unpadded) token layout: the tails of a batch of requests, each with its own
+ * resume point, back to back in one launch, as an engine batches them (the
+ * paper's engine schedules the resumed tail of every request, Section 2.2).
+ *
+ * Identical to hs_linattn_prefill_from_state (same arithmetic, same bits)
+ * except where each problem's tokens live: token t of problem b is row
+ * cu_rows[b] + t of q, k, v, log_g and o, which are [rows][n_heads][d]; the
+ * shape's max_tokens is not used.
+ *   cu_rows  host int64 [batch + 1], 0 <= cu_rows[b] <= cu_rows[b+1] and
+ *            n_tokens[b] <= cu_rows[b+1] - cu_rows[b] (the usual cumulative
+ *            sequence lengths have equality); rows must stay below 2^31
+ * Errors: as hs_linattn_prefill_from_state; HS_ERR_INVALID_ARG also for a NULL
+ * or non-monotone cu_rows or a problem longer than its rows.
+ */
+hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t *q,
+                                    const uint16_t *k, const uint16_t *v, const float *log_g,
+                                    float *o, float *state, const int64_t *pos0,
+                                    const int32_t *n_tokens, const int64_t *cu_rows,
+                                    int32_t ckpt_interval, float *const *ckpt_slots,
+                                    int32_t *d_err, cudaStream_t stream);
 
 /*
  * hs_linattn_num_checkpoints -- number of checkpoint slots the prefill above

@@ -31,7 +31,7 @@ HS_DEVERR_MISALIGNED = 2
 HS_DEVERR_NULL = 3
 HS_DEVERR_TIMEOUT = 4
 
-HS_MAX_BATCH = 512
+HS_MAX_BATCH = 384
 HS_CHUNK = 64
 HS_SHORT_SEGMENT = 8
 
@@ -43,7 +43,7 @@ HS_LINATTN_SINGLE_TOKEN = 3
 EXPORTED = ("hs_status_string", "hs_version", "hs_align_prefix", "hs_restore_kv_pages",
             "hs_save_kv_pages", "hs_restore_kv_page_slices", "hs_save_kv_page_slices",
             "hs_restore_state", "hs_checkpoint_states", "hs_linattn_prefill_from_state",
-            "hs_linattn_num_checkpoints")
+            "hs_linattn_num_checkpoints", "hs_linattn_prefill_packed")
 
 
 class HsError(RuntimeError):
@@ -86,6 +86,8 @@ def load() -> C.CDLL:
             L.hs_linattn_prefill_from_state.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp,
                                                         vp, vp, vp, vp, vp, i32, vp, vp, vp]
             L.hs_linattn_num_checkpoints.argtypes = [i32, vp, vp, i32, vp]
+            L.hs_linattn_prefill_packed.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp, vp,
+                                                    vp, vp, vp, vp, vp, i32, vp, vp, vp]
             for name in EXPORTED[2:]:
                 getattr(L, name).restype = C.c_int
             _lib = L
@@ -210,6 +212,22 @@ def hs_linattn_prefill_from_state(shape: hs_linattn_shape, q, k, v, log_g, o, st
                                               int(ckpt_interval), _ptr(ckpt_slots), _ptr(d_err),
                                               _stream(stream))
     _check(rc, "hs_linattn_prefill_from_state")
+
+
+def hs_linattn_prefill_packed(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0, n_tokens,
+                              cu_rows, ckpt_interval: int, ckpt_slots=None, d_err=None,
+                              stream=None):
+    """Packed token layout: token t of problem b is row cu_rows[b] + t.  pos0 / n_tokens /
+    cu_rows: host sequences of length batch, batch, batch + 1."""
+    B = int(shape.batch)
+    p0 = (C.c_int64 * max(B, 1))(*[int(x) for x in pos0])
+    nt = (C.c_int32 * max(B, 1))(*[int(x) for x in n_tokens])
+    cu = (C.c_int64 * max(B + 1, 1))(*[int(x) for x in cu_rows])
+    rc = load().hs_linattn_prefill_packed(C.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(log_g),
+                                          _ptr(o), _ptr(state), C.addressof(p0), C.addressof(nt),
+                                          C.addressof(cu), int(ckpt_interval), _ptr(ckpt_slots),
+                                          _ptr(d_err), _stream(stream))
+    _check(rc, "hs_linattn_prefill_packed")
 
 
 def hs_linattn_num_checkpoints(pos0, n_tokens, ckpt_interval: int) -> int:

@@ -525,7 +525,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     auto prefetch = [&](int64_t t) {
         if (t >= n)
             return;
-        const int32_t y = (int32_t)((int64_t)b * p.max_tokens + t);
+        const int32_t y = (int32_t)((int64_t)p.row0[b] + t);
         const int32_t x = h * D;
         tma_prefetch_2d(&maps.q, x, y);
         tma_prefetch_2d(&maps.k, x, y);
@@ -536,7 +536,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // first start on the 64-token grid, so the segment kPrefetch ahead starts at
     // tok_local + 64 * kPrefetch and is requested into L2 now
     auto issue_tma = [&](int64_t tok_local) {
-        const int32_t y = (int32_t)((int64_t)b * p.max_tokens + tok_local);
+        const int32_t y = (int32_t)((int64_t)p.row0[b] + tok_local);
         const int32_t x = h * D;
         mbar_arrive_expect_tx(bar_tma, STAGE_BYTES);
         tma_load_2d(sb + OFF_SQ, &maps.q, x, y, bar_tma);
@@ -681,7 +681,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         __syncthreads();
         if (tid == kIssuer && seg_end < end)
             issue_tma(tok_s + L);
-        float *ob = p.o + (((int64_t)b * p.max_tokens + tok_s) * p.n_heads + h) * D;
+        float *ob = p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D;
         for (int idx = tid; idx < L * D; idx += NT) {
             const int i = idx >> 7, e = idx & (D - 1);
             float sum = part[(i * 8) * D + e];
@@ -833,7 +833,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (!wait_all(bar_s, ph_s))
             return false;
         state_pass(smem, tmem, -1, ckpt_slot(seg_end), false);   // checkpoint and |S| of the final state
-        out_epilogue(tmem, p.o + (((int64_t)b * p.max_tokens + tok_s) * p.n_heads + h) * D, tstride, L, par);
+        out_epilogue(tmem, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride, L, par);
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -853,7 +853,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // ---- long segments: fast ones pipelined two deep, exact ones one at a time
     {
         const auto out_of = [&](int64_t t) {
-            return p.o + (((int64_t)b * p.max_tokens + t) * p.n_heads + h) * D;
+            return p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D;
         };
         int par = 0;
         bool have_prep = false, prep_fast = false, qk_issued = false;
@@ -1062,22 +1062,25 @@ bool encode_rows(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint6
 
 }  // namespace
 
-bool gla_chunked_tc_supported(int d, int64_t batch, int64_t max_tokens)
+bool gla_chunked_tc_supported(int d)
 {
-    return d == D && batch * max_tokens < ((int64_t)1 << 31);
+    return d == D;
 }
 
 cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s)
 {
-    if (!gla_chunked_tc_supported(d, p.batch, p.max_tokens))
+    if (!gla_chunked_tc_supported(d))
         return cudaErrorNotSupported;
     TmaMaps maps;
     const uint64_t inner = (uint64_t)p.n_heads * D;
-    // rows up to the last problem's last token: copies never read beyond the tokens the
+    // rows up to the last token any problem has: copies never read beyond the tokens the
     // caller passed (boxes reaching further are zero-filled), so q/k/v/log_g may be
-    // offset views whose batch stride runs past the end of the allocation
-    const uint64_t rows = (uint64_t)(p.batch - 1) * (uint64_t)p.max_tokens +
-                          (uint64_t)p.n_tokens[p.batch - 1];
+    // offset views whose last rows run past the end of the allocation
+    uint64_t rows = 0;
+    for (int32_t b = 0; b < p.batch; ++b) {
+        const uint64_t r = (uint64_t)p.row0[b] + (uint64_t)p.n_tokens[b];
+        rows = r > rows ? r : rows;
+    }
     if (rows == 0)
         return cudaSuccess;
     if (!encode_rows(&maps.q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.q, inner, rows, 2) ||

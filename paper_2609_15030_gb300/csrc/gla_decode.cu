@@ -51,7 +51,7 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __
     for (int r = 0; r < 16; ++r)
         S[r] = *reinterpret_cast<const float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg);
 
-    const int64_t row = ((int64_t)b * p.max_tokens) * p.n_heads + h;   // the call's one token
+    const int64_t row = ((int64_t)p.row0[b]) * p.n_heads + h;   // the call's one token
     const uint4 *q8 = reinterpret_cast<const uint4 *>(p.q + row * D + 16 * rg);
     const uint4 *k8 = reinterpret_cast<const uint4 *>(p.k + row * D + 16 * rg);
     const float4 *a4 = reinterpret_cast<const float4 *>(p.log_g + row * D + 16 * rg);

@@ -62,7 +62,7 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_recurrent_kernel(const
         const int tb = min(kTokBlock, n - t0);
         for (int idx = tid; idx < tb * D; idx += NTH) {
             const int tt = idx / D, d = idx - (idx / D) * D;
-            const int64_t row = ((int64_t)b * p.max_tokens + t0 + tt) * p.n_heads + h;
+            const int64_t row = ((int64_t)p.row0[b] + t0 + tt) * p.n_heads + h;
             sq[tt][d] = bf16_to_f32(p.q[row * D + d]);
             sk[tt][d] = bf16_to_f32(p.k[row * D + d]);
             sv[tt][d] = bf16_to_f32(p.v[row * D + d]);
@@ -119,7 +119,7 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_recurrent_kernel(const
 #pragma unroll
             for (int g = 1; g < NRG; ++g)
                 sum += spart[tt][g][e];
-            const int64_t row = ((int64_t)b * p.max_tokens + t0 + tt) * p.n_heads + h;
+            const int64_t row = ((int64_t)p.row0[b] + t0 + tt) * p.n_heads + h;
             p.o[row * D + e] = sum;
         }
         __syncthreads();

@@ -230,12 +230,13 @@ hs_status hs_linattn_num_checkpoints(int32_t batch, const int64_t *pos0, const i
     return HS_OK;
 }
 
-hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint16_t *q,
-                                        const uint16_t *k, const uint16_t *v, const float *log_g,
-                                        float *o, float *state, const int64_t *pos0,
-                                        const int32_t *n_tokens, int32_t ckpt_interval,
-                                        float *const *ckpt_slots, int32_t *d_err,
-                                        cudaStream_t stream)
+// The prefill of both token layouts: cu_rows == nullptr is the padded layout (problem b's
+// token t at row b*max_tokens + t), else problem b's token t is at row cu_rows[b] + t.
+static hs_status prefill(const hs_linattn_shape *shp, const uint16_t *q, const uint16_t *k,
+                         const uint16_t *v, const float *log_g, float *o, float *state,
+                         const int64_t *pos0, const int32_t *n_tokens, const int64_t *cu_rows,
+                         int32_t ckpt_interval, float *const *ckpt_slots, int32_t *d_err,
+                         cudaStream_t stream)
 {
     if (shp == nullptr)
         return HS_ERR_INVALID_ARG;
@@ -259,10 +260,17 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
         return HS_ERR_INVALID_ARG;
     bool any_tokens = false;
     for (int32_t b = 0; b < s.batch; ++b) {
-        if (pos0[b] < 0 || n_tokens[b] < 0 || (int64_t)n_tokens[b] > s.max_tokens)
+        if (pos0[b] < 0 || n_tokens[b] < 0)
             return HS_ERR_INVALID_ARG;
         if (pos0[b] > ((int64_t)1 << 40))
             return HS_ERR_INVALID_ARG;
+        if (cu_rows == nullptr) {
+            if ((int64_t)n_tokens[b] > s.max_tokens)
+                return HS_ERR_INVALID_ARG;
+        } else if (cu_rows[b] < 0 || cu_rows[b + 1] < cu_rows[b] ||
+                   (int64_t)n_tokens[b] > cu_rows[b + 1] - cu_rows[b]) {
+            return HS_ERR_INVALID_ARG;
+        }
         any_tokens = any_tokens || n_tokens[b] > 0;
     }
     if (!any_tokens)
@@ -283,14 +291,17 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
     p.state = state;
     p.ckpt_slots = (ckpt_interval > 0) ? ckpt_slots : nullptr;
     p.d_err = d_err;
-    p.max_tokens = s.max_tokens;
     p.batch = s.batch;
     p.n_heads = s.n_heads;
     p.ckpt_interval = (p.ckpt_slots != nullptr) ? ckpt_interval : 0;
     int64_t base = 0;
     for (int32_t b = 0; b < s.batch; ++b) {
+        const int64_t r0 = cu_rows ? cu_rows[b] : (int64_t)b * s.max_tokens;
+        if (r0 + n_tokens[b] > INT32_MAX)
+            return HS_ERR_UNSUPPORTED;   // token rows are 32-bit
         p.pos0[b] = pos0[b];
         p.n_tokens[b] = n_tokens[b];
+        p.row0[b] = (int32_t)r0;
         p.ck_base[b] = (int32_t)base;
         if (p.ckpt_interval > 0 && n_tokens[b] > 0)
             base += (pos0[b] + n_tokens[b]) / p.ckpt_interval - pos0[b] / p.ckpt_interval;
@@ -298,7 +309,7 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
     if (base > INT32_MAX)
         return HS_ERR_INVALID_ARG;
 
-    const bool tc_ok = hs::gla_chunked_tc_supported(s.d_k, s.batch, s.max_tokens);
+    const bool tc_ok = hs::gla_chunked_tc_supported(s.d_k);
     if (s.kernel == HS_LINATTN_CHUNKED_TC && !tc_ok)
         return HS_ERR_UNSUPPORTED;
     int32_t max_n = 0;
@@ -317,6 +328,30 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
     if (s.kernel == HS_LINATTN_SINGLE_TOKEN || (s.kernel == HS_LINATTN_AUTO && max_n == 1))
         return cuda_status(hs::launch_gla_decode(p, s.d_k, stream));
     return cuda_status(hs::launch_gla_recurrent(p, s.d_k, stream));
+}
+
+hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint16_t *q,
+                                        const uint16_t *k, const uint16_t *v, const float *log_g,
+                                        float *o, float *state, const int64_t *pos0,
+                                        const int32_t *n_tokens, int32_t ckpt_interval,
+                                        float *const *ckpt_slots, int32_t *d_err,
+                                        cudaStream_t stream)
+{
+    return prefill(shp, q, k, v, log_g, o, state, pos0, n_tokens, nullptr, ckpt_interval,
+                   ckpt_slots, d_err, stream);
+}
+
+hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t *q,
+                                    const uint16_t *k, const uint16_t *v, const float *log_g,
+                                    float *o, float *state, const int64_t *pos0,
+                                    const int32_t *n_tokens, const int64_t *cu_rows,
+                                    int32_t ckpt_interval, float *const *ckpt_slots,
+                                    int32_t *d_err, cudaStream_t stream)
+{
+    if (shp != nullptr && shp->batch > 0 && cu_rows == nullptr)
+        return HS_ERR_INVALID_ARG;
+    return prefill(shp, q, k, v, log_g, o, state, pos0, n_tokens, cu_rows, ckpt_interval,
+                   ckpt_slots, d_err, stream);
 }
 
 }  // extern "C"

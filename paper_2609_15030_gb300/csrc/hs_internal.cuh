@@ -54,14 +54,13 @@ struct GlaParams {
     float *state;
     float *const *ckpt_slots;  // device array or nullptr
     int32_t *d_err;
-    int64_t max_tokens;
     int32_t batch;
     int32_t n_heads;
     int32_t ckpt_interval;     // 0: none
-    int32_t pad_;
     int64_t pos0[HS_MAX_BATCH];
     int32_t n_tokens[HS_MAX_BATCH];
     int32_t ck_base[HS_MAX_BATCH];  // index of the problem's first slot in ckpt_slots
+    int32_t row0[HS_MAX_BATCH];     // token row of the problem's first token in q/k/v/log_g/o
 };
 
 // launchers (return the launch's cudaError_t)
@@ -80,6 +79,6 @@ cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t
 cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_decode(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s);
-bool gla_chunked_tc_supported(int d, int64_t batch, int64_t max_tokens);
+bool gla_chunked_tc_supported(int d);
 
 }  // namespace hs

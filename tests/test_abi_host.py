@@ -4,6 +4,7 @@
 * hs_align_prefix (host integer code) matches the oracle bit-exactly;
 * every argument error is reported before any CUDA call.
 """
+import ctypes
 import os
 import re
 
@@ -172,7 +173,8 @@ def test_prefill_host_validation():
     cases = [
         (dict(shape_kw=dict(d_k=96, d_v=96)), hs.HS_ERR_UNSUPPORTED),
         (dict(shape_kw=dict(d_k=64, d_v=128)), hs.HS_ERR_UNSUPPORTED),
-        (dict(shape_kw=dict(batch=hs.HS_MAX_BATCH + 1), pos0=[0] * 513, n_tokens=[1] * 513),
+        (dict(shape_kw=dict(batch=hs.HS_MAX_BATCH + 1), pos0=[0] * (hs.HS_MAX_BATCH + 1),
+          n_tokens=[1] * (hs.HS_MAX_BATCH + 1)),
          hs.HS_ERR_UNSUPPORTED),
         (dict(ckpt_interval=96), hs.HS_ERR_UNSUPPORTED),
         (dict(ckpt_interval=-64), hs.HS_ERR_INVALID_ARG),
@@ -193,6 +195,32 @@ def test_prefill_host_validation():
         assert e.value.status == code, kw
     call(shape_kw=dict(batch=0), pos0=[], n_tokens=[])    # empty batch: OK, nothing launched
     call(n_tokens=[0], q=None, k=None, v=None, log_g=None, o=None)   # empty tails: OK
+
+
+def test_packed_prefill_host_validation():
+    def call(**kw):
+        a = dict(q=FAKE, k=FAKE, v=FAKE, log_g=FAKE, o=FAKE, state=FAKE, pos0=[0, 5],
+                 n_tokens=[8, 3], cu_rows=[0, 8, 11], ckpt_interval=64, ckpt_slots=None,
+                 d_err=None, stream=0)
+        a.update(kw)
+        hs.hs_linattn_prefill_packed(hs.make_shape(2, 2, 64, 64, 0), **a)
+    for kw, code in [(dict(cu_rows=[0, 8, 10]), hs.HS_ERR_INVALID_ARG),     # problem 1 too long
+                     (dict(cu_rows=[0, 12, 11]), hs.HS_ERR_INVALID_ARG),    # not monotone
+                     (dict(cu_rows=[-1, 8, 11]), hs.HS_ERR_INVALID_ARG),
+                     (dict(cu_rows=[0, 2 ** 31 - 2, 2 ** 31 + 8]), hs.HS_ERR_UNSUPPORTED),
+                     (dict(n_tokens=[9, 3]), hs.HS_ERR_INVALID_ARG)]:
+        with pytest.raises(hs.HsError) as e:
+            call(**kw)
+        assert e.value.status == code, kw
+    lib = hs.load()
+    shape = hs.make_shape(2, 2, 64, 64, 0)
+    p0 = (ctypes.c_int64 * 2)(0, 5)
+    nt = (ctypes.c_int32 * 2)(8, 3)
+    rc = lib.hs_linattn_prefill_packed(ctypes.byref(shape), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE,
+                                       ctypes.addressof(p0), ctypes.addressof(nt), None, 64, None,
+                                       None, None)
+    assert rc == hs.HS_ERR_INVALID_ARG                       # cu_rows is required
+    call(n_tokens=[0, 0], q=None, k=None, v=None, log_g=None, o=None)   # empty tails: OK
 
 
 def test_missing_library_fails_loudly(monkeypatch, tmp_path):

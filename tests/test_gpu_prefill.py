@@ -425,3 +425,60 @@ def test_offset_views_read_only_the_given_tokens(kernel):
     assert np.array_equal(got[:, c:].view(np.uint32), o_ref[:, :T - c].view(np.uint32))
     assert (got[:, :c] == 7.0).all()
     assert np.array_equal(state.cpu().numpy().view(np.uint32), S_ref.view(np.uint32))
+
+
+@pytest.mark.parametrize("kernel", KERNELS + [pytest.param(hs.HS_LINATTN_AUTO, id="auto")])
+def test_packed_layout_equals_padded_bitwise(kernel):
+    """A batch of tails with different resume points and lengths (0, ragged, several chunks),
+    packed back to back without padding, gives the padded layout's outputs, final states and
+    checkpoints bit for bit, and those follow the oracle."""
+    dev = device()
+    nH, d, T, C = 4, 128, 200, 64
+    pos0 = [64, 0, 4093, 700, 130]
+    n_tok = [200, 0, 37, 129, 5]
+    B = len(pos0)
+    inp = gen_linear(31, 0, B, T, nH, d, d)
+    S0 = gen_state(31, 0, B, nH, d, d)
+    o_pad, S_pad, ck_pad = run_prefill(inp, pos0, n_tok, S0, C, dev, kernel)
+    cu = [0]
+    for n in n_tok:
+        cu.append(cu[-1] + n)
+    cat = lambda x: np.concatenate([x[b, :n_tok[b]] for b in range(B)], axis=0)[None]
+    q, k, v, a = (to_dev(cat(x), dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    state = to_dev(np.asarray(S0, np.float32), dev)
+    o = torch.full((cu[-1], nH, d), float("nan"), device=dev)
+    nck = hs.hs_linattn_num_checkpoints(pos0, n_tok, C)
+    slots = torch.full((nck, nH, d, d), float("nan"), device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_linattn_prefill_packed(hs.make_shape(B, nH, d, d, 0, kernel), q, k, v, a, o, state,
+                                 pos0, n_tok, cu, C, hs.ptr_array([slots[i] for i in range(nck)], dev),
+                                 err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    o_p = o.cpu().numpy()
+    for b in range(B):
+        assert np.array_equal(o_p[cu[b]:cu[b + 1]].view(np.uint32), o_pad[b, :n_tok[b]].view(np.uint32))
+    assert np.array_equal(state.cpu().numpy().view(np.uint32), S_pad.view(np.uint32))
+    assert np.array_equal(slots.cpu().numpy().view(np.uint32),
+                          np.concatenate(ck_pad, axis=0).view(np.uint32))
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, pos0, n_tok, S0=S0, C_=C)
+    _check(o_pad, S_pad, ck_pad, ro, rS, rck, pos0, n_tok, "packed")
+
+
+def test_packed_decode_steps_match_padded():
+    """One token per problem from a packed layout (cu_rows = 0..B) through the single-token
+    kernel equals the padded call bit for bit."""
+    dev = device()
+    nH, d, B = 8, 128, 6
+    inp = gen_linear(32, 0, B, 1, nH, d, d)
+    S0 = gen_state(32, 0, B, nH, d, d)
+    pos0 = [10, 63, 127, 4000, 2, 511]
+    o_pad, S_pad, _ = run_prefill(inp, pos0, [1] * B, S0, 64, dev, hs.HS_LINATTN_SINGLE_TOKEN)
+    q, k, v, a = (to_dev(x.reshape(1, B, nH, d), dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    state = to_dev(np.asarray(S0, np.float32), dev)
+    o = torch.empty((B, nH, d), device=dev)
+    hs.hs_linattn_prefill_packed(hs.make_shape(B, nH, d, d, 0, hs.HS_LINATTN_SINGLE_TOKEN), q, k,
+                                 v, a, o, state, pos0, [1] * B, list(range(B + 1)), 0)
+    torch.cuda.synchronize()
+    assert np.array_equal(o.cpu().numpy().view(np.uint32), o_pad[:, 0].view(np.uint32))
+    assert np.array_equal(state.cpu().numpy().view(np.uint32), S_pad.view(np.uint32))
