@@ -908,14 +908,14 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             if (tid == kIssuer) {
                 tc_fence_after();
                 if (!qk_issued) {
-#pragma unroll
+#pragma unroll 1
                     for (int kk = 0; kk < D / 16; ++kk) {
                         const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
                         mma_f16_ss(tmem + TM_A, sdesc_sw128(setb + S_QH + koff, 16, 1024),
                                    sdesc_sw128(setb + S_KH + koff, 16, 1024), IDF_N64, kk > 0);
                     }
                 }
-#pragma unroll
+#pragma unroll 1
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
                     mma_f16_ts(tmem + (par ? TM_O1 : TM_O0), tmem + TM_SH + kk * 8,
@@ -950,14 +950,14 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             if (tid == kIssuer) {
                 tc_fence_after();
                 const uint32_t vt = tmem + TM_V + 32 * par;
-#pragma unroll
+#pragma unroll 1
                 for (int kk = 0; kk < CH / 16; ++kk)
                     mma_f16_ts(tmem + (par ? TM_S : TM_O0), vt + kk * 8,
                                sdesc_sw128(setb + S_B2H + kk * 32, 16, 1024), IDF_N192, 1);
                 tc_commit(bar_o);
                 if (next_fast) {
                     const uint32_t nsetb = sb + (uint32_t)(par ^ 1) * SET_BYTES;
-#pragma unroll
+#pragma unroll 1
                     for (int kk = 0; kk < D / 16; ++kk) {
                         const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
                         mma_f16_ss(tmem + TM_A, sdesc_sw128(nsetb + S_QH + koff, 16, 1024),
