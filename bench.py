@@ -80,7 +80,7 @@ def kv_bytes(n_layers, n_pages, page_bytes):
 
 
 KERNEL_OF = {"decode": "gla_decode_kernel<128>", "prefill": "gla_chunked_tc_kernel",
-             "restore": "kv_scatter_kernel+slot_copy_kernel"}
+             "restore": "restore_request_kernel"}
 
 
 def _traffic():
@@ -211,13 +211,10 @@ class Hybrid12:
     def phase_restore(self, s, r, st):
         """KV page restore of [0,c) for the full layers + state restore at c."""
         hs, R, I, O = self.hs, self.req[r], self.inp[(s, r)], self.out[r]
-        n = 0
-        if R["n_pages"]:
-            hs.hs_restore_kv_pages(I["staging_ptrs"], self.cache_ptrs, self.nF, I["bt"],
-                                   R["n_pages"], self.page_bytes, self.NB, None, st)
-            n += 1
-        hs.hs_restore_state(I["ck_ptrs"], O["live_ptrs"], self.nL, self.state_floats, None, st)
-        return n + 1
+        hs.hs_restore_request(I["staging_ptrs"], self.cache_ptrs, self.nF, I["bt"], R["n_pages"],
+                              self.page_bytes, self.NB, I["ck_ptrs"], O["live_ptrs"], self.nL,
+                              self.state_floats, None, st)
+        return 1
 
     def phase_prefill(self, s, r, st):
         """Tail prefill of [c,L) for all linear layers, emitting the checkpoint at L."""
@@ -879,9 +876,9 @@ def run_long(dev):
             slot_ptrs = hs.ptr_array([slots[b] for b in range(B)], dev) if L % C == 0 else None
             tok = c * nH * d
             def resume():
-                for b in range(B):
-                    hs.hs_restore_kv_pages(stg_ptrs[b], cache_ptrs, nF, bts[b], n_pages, pb, NB)
-                hs.hs_restore_state(src_ptrs, dst_ptrs, nL, B * nH * d * d)
+                for b in range(B):      # the batch's states ride with the first request's pages
+                    hs.hs_restore_request(stg_ptrs[b], cache_ptrs, nF, bts[b], n_pages, pb, NB,
+                                          src_ptrs, dst_ptrs, nL if b == 0 else 0, B * nH * d * d)
                 for l in range(nL):
                     hs.hs_linattn_prefill_from_state(
                         shape_t, q.data_ptr() + 2 * tok, k.data_ptr() + 2 * tok, v.data_ptr() + 2 * tok,

@@ -131,6 +131,29 @@ hs_status hs_restore_kv_pages(const void *const *staging_layers, void *const *ca
                               cudaStream_t stream);
 
 /*
+ * hs_restore_request -- hs_restore_kv_pages and hs_restore_state of one resumed
+ * request in a single launch.
+ *
+ * Paper: Section 2.1 and Section 5.2 (the attention cache entries of [0,B) are
+ * restored together with the recurrent state at B), Section 1 and Section 2.2.
+ *
+ * Same effect as hs_restore_kv_pages(staging_layers, cache_layers, n_layers,
+ * block_table, n_pages, page_bytes, num_blocks) followed by
+ * hs_restore_state(src_slots, dst_slots, n_slots, floats_each), with every slot
+ * pointer 16-byte aligned (else HS_DEVERR_MISALIGNED and that slot is skipped)
+ * and floats_each a multiple of 4.  The restored states are written so that a
+ * prefill launched next finds them in L2.  Either part may be empty (n_layers or
+ * n_pages == 0; n_slots or floats_each == 0).
+ * Errors: HS_ERR_INVALID_ARG, HS_ERR_MISALIGNED (page_bytes % 16, floats_each % 4),
+ * HS_ERR_CUDA.
+ */
+hs_status hs_restore_request(const void *const *staging_layers, void *const *cache_layers,
+                             int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                             int64_t page_bytes, int64_t num_blocks, const float *const *src_slots,
+                             float *const *dst_slots, int32_t n_slots, int64_t floats_each,
+                             int32_t *d_err, cudaStream_t stream);
+
+/*
  * hs_save_kv_pages -- gather KV pages of the paged cache into a staging pool (save).
  *
  * Paper: Section 3.1 (a save must have completed, not merely been submitted,

@@ -43,7 +43,7 @@ HS_LINATTN_SINGLE_TOKEN = 3
 EXPORTED = ("hs_status_string", "hs_version", "hs_align_prefix", "hs_restore_kv_pages",
             "hs_save_kv_pages", "hs_restore_kv_page_slices", "hs_save_kv_page_slices",
             "hs_restore_state", "hs_checkpoint_states", "hs_linattn_prefill_from_state",
-            "hs_linattn_num_checkpoints", "hs_linattn_prefill_packed")
+            "hs_linattn_num_checkpoints", "hs_linattn_prefill_packed", "hs_restore_request")
 
 
 class HsError(RuntimeError):
@@ -79,6 +79,7 @@ def load() -> C.CDLL:
             L.hs_align_prefix.argtypes = [i64, i64, vp, i32, i32, vp, vp, vp]
             L.hs_restore_kv_pages.argtypes = [vp, vp, i32, vp, i32, i64, i64, vp, vp]
             L.hs_save_kv_pages.argtypes = [vp, vp, i32, vp, i32, i64, i64, vp, vp]
+            L.hs_restore_request.argtypes = [vp, vp, i32, vp, i32, i64, i64, vp, vp, i32, i64, vp, vp]
             for name in ("hs_restore_kv_page_slices", "hs_save_kv_page_slices"):
                 getattr(L, name).argtypes = [vp, vp, i32, vp, i32, i64, i32, i64, i64, i64, vp, vp]
             L.hs_restore_state.argtypes = [vp, vp, i32, i64, vp, vp]
@@ -151,6 +152,16 @@ def hs_restore_kv_pages(staging_layers, cache_layers, n_layers: int, block_table
                                     _ptr(block_table), int(n_pages), int(page_bytes),
                                     int(num_blocks), _ptr(d_err), _stream(stream))
     _check(rc, "hs_restore_kv_pages")
+
+
+def hs_restore_request(staging_layers, cache_layers, n_layers: int, block_table, n_pages: int,
+                       page_bytes: int, num_blocks: int, src_slots, dst_slots, n_slots: int,
+                       floats_each: int, d_err=None, stream=None):
+    rc = load().hs_restore_request(_ptr(staging_layers), _ptr(cache_layers), int(n_layers),
+                                   _ptr(block_table), int(n_pages), int(page_bytes),
+                                   int(num_blocks), _ptr(src_slots), _ptr(dst_slots), int(n_slots),
+                                   int(floats_each), _ptr(d_err), _stream(stream))
+    _check(rc, "hs_restore_request")
 
 
 def hs_save_kv_pages(cache_layers, staging_layers, n_layers: int, block_table, n_pages: int,

@@ -19,6 +19,11 @@
 namespace hs {
 namespace {
 
+__device__ __forceinline__ void prefetch_l2(const void *p)
+{
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ float bf16_lo(uint32_t w)
 {
     return __uint_as_float(w << 16);
@@ -40,10 +45,22 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __
     if (p.n_tokens[b] <= 0)
         return;
     const int64_t pos0 = p.pos0[b];
-    pdl_wait_and_release();
     const int tid = threadIdx.x;
     const int cg = tid % NCG;
     const int rg = tid / NCG;
+    {
+        const int64_t prow = ((int64_t)p.row0[b]) * p.n_heads + h;
+        constexpr int LB = D / 64;     // 128-byte lines of one bf16 row (a float row is 2 LB)
+        if (tid < LB)
+            prefetch_l2(reinterpret_cast<const char *>(p.q + prow * D) + 128 * tid);
+        else if (tid < 2 * LB)
+            prefetch_l2(reinterpret_cast<const char *>(p.k + prow * D) + 128 * (tid - LB));
+        else if (tid < 3 * LB)
+            prefetch_l2(reinterpret_cast<const char *>(p.v + prow * D) + 128 * (tid - 2 * LB));
+        else if (tid < 5 * LB)
+            prefetch_l2(reinterpret_cast<const char *>(p.log_g + prow * D) + 128 * (tid - 3 * LB));
+    }
+    pdl_wait_and_release();
 
     float *st = p.state + ((int64_t)b * p.n_heads + h) * D * D;
     float4 S[16];

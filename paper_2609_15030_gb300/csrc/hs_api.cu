@@ -199,6 +199,37 @@ hs_status hs_save_kv_page_slices(const void *const *cache_layers, void *const *s
                      page_bytes, rows, col_off, col_bytes, num_blocks, d_err, stream);
 }
 
+hs_status hs_restore_request(const void *const *staging_layers, void *const *cache_layers,
+                             int32_t n_layers, const int32_t *block_table, int32_t n_pages,
+                             int64_t page_bytes, int64_t num_blocks, const float *const *src_slots,
+                             float *const *dst_slots, int32_t n_slots, int64_t floats_each,
+                             int32_t *d_err, cudaStream_t stream)
+{
+    if (n_layers < 0 || n_pages < 0 || page_bytes <= 0 || num_blocks < 0 || n_slots < 0 ||
+        floats_each < 0)
+        return HS_ERR_INVALID_ARG;
+    if (page_bytes % 16 != 0 || floats_each % 4 != 0)
+        return HS_ERR_MISALIGNED;
+    const bool kv = n_layers > 0 && n_pages > 0;
+    const bool st = n_slots > 0 && floats_each > 0;
+    if (kv && (staging_layers == nullptr || cache_layers == nullptr || block_table == nullptr))
+        return HS_ERR_INVALID_ARG;
+    if (kv && (int64_t)n_pages > num_blocks)
+        return HS_ERR_INVALID_ARG;  // a request's pages occupy distinct blocks
+    if (st && (src_slots == nullptr || dst_slots == nullptr))
+        return HS_ERR_INVALID_ARG;
+    if (!kv && !st)
+        return HS_OK;
+    int sms = 0;
+    hs_status status = sm_count(&sms);
+    if (status != HS_OK)
+        return status;
+    return cuda_status(hs::launch_restore_request(
+        staging_layers, cache_layers, kv ? n_layers : 0, block_table, kv ? n_pages : 0, page_bytes,
+        num_blocks, src_slots, dst_slots, st ? n_slots : 0, st ? floats_each : 0, d_err, sms,
+        stream));
+}
+
 hs_status hs_restore_state(const float *const *src_slots, float *const *dst_slots, int32_t n,
                            int64_t floats_each, int32_t *d_err, cudaStream_t stream)
 {

@@ -74,6 +74,11 @@ cudaError_t launch_kv_slices(bool gather, const void *const *from, void *const *
                              const int32_t *bt, int32_t n_pages, int64_t page_bytes, int32_t rows,
                              int64_t col_off, int64_t col_bytes, int64_t num_blocks, int32_t *d_err,
                              int sm_count, cudaStream_t s);
+cudaError_t launch_restore_request(const void *const *staging, void *const *cache, int32_t n_layers,
+                                   const int32_t *bt, int32_t n_pages, int64_t page_bytes,
+                                   int64_t num_blocks, const float *const *src_slots,
+                                   float *const *dst_slots, int32_t n_slots, int64_t floats_each,
+                                   int32_t *d_err, int sm_count, cudaStream_t s);
 cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t n,
                              int64_t floats_each, int32_t *d_err, int sm_count, cudaStream_t s);
 cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);

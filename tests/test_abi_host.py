@@ -152,6 +152,31 @@ def test_kv_page_slices_host_validation(fn):
     call(n_pages=0)
 
 
+def test_restore_request_host_validation():
+    def call(**kw):
+        a = dict(staging_layers=FAKE, cache_layers=FAKE, n_layers=1, block_table=FAKE, n_pages=1,
+                 page_bytes=64, num_blocks=4, src_slots=FAKE, dst_slots=FAKE, n_slots=2,
+                 floats_each=16, d_err=None, stream=0)
+        a.update(kw)
+        hs.hs_restore_request(**a)
+    for kw, code in [(dict(n_layers=-1), hs.HS_ERR_INVALID_ARG),
+                     (dict(n_slots=-1), hs.HS_ERR_INVALID_ARG),
+                     (dict(floats_each=-4), hs.HS_ERR_INVALID_ARG),
+                     (dict(page_bytes=0), hs.HS_ERR_INVALID_ARG),
+                     (dict(page_bytes=24), hs.HS_ERR_MISALIGNED),
+                     (dict(floats_each=18), hs.HS_ERR_MISALIGNED),
+                     (dict(staging_layers=None), hs.HS_ERR_INVALID_ARG),
+                     (dict(block_table=None), hs.HS_ERR_INVALID_ARG),
+                     (dict(src_slots=None), hs.HS_ERR_INVALID_ARG),
+                     (dict(n_pages=5, num_blocks=4), hs.HS_ERR_INVALID_ARG)]:
+        with pytest.raises(hs.HsError) as e:
+            call(**kw)
+        assert e.value.status == code, kw
+    # both parts empty: OK without touching the GPU (a missing part's pointers are not read)
+    call(n_layers=0, n_slots=0)
+    call(n_pages=0, staging_layers=None, floats_each=0, src_slots=None)
+
+
 def test_state_copy_host_validation():
     for fn in (hs.hs_restore_state, hs.hs_checkpoint_states):
         with pytest.raises(hs.HsError):

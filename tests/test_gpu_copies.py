@@ -176,3 +176,118 @@ def test_scatter_from_pinned_host_staging():
     mask = torch.ones(nb, dtype=torch.bool)
     mask[bt.long().cpu()] = False
     assert bool((c[:, mask] == POISON).all())
+
+
+def _request_case(dev, n_layers, n_pages, page_bytes, num_blocks, n_slots, floats_each, seed):
+    staging = [gen_kv_pages(seed, l, n_pages, page_bytes) for l in range(n_layers)]
+    bt = gen_block_table(seed, 0, n_pages, num_blocks)
+    rng = np.random.default_rng(seed)
+    src_h = [rng.standard_normal(floats_each).astype(np.float32) for _ in range(n_slots)]
+    d_st = [torch.from_numpy(s.reshape(-1)).to(dev) for s in staging]
+    d_cache = [torch.full((num_blocks * page_bytes,), POISON, dtype=torch.uint8, device=dev)
+               for _ in range(n_layers)]
+    src = [torch.from_numpy(x).to(dev) for x in src_h]
+    dst = [torch.full((floats_each,), -7.0, device=dev) for _ in range(n_slots)]
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_restore_request(hs.ptr_array(d_st, dev), hs.ptr_array(d_cache, dev), n_layers,
+                          torch.from_numpy(bt).to(dev), n_pages, page_bytes, num_blocks,
+                          hs.ptr_array(src, dev), hs.ptr_array(dst, dev), n_slots, floats_each, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    h_cache = [np.full(num_blocks * page_bytes, POISON, np.uint8) for _ in range(n_layers)]
+    if n_pages:
+        oracle.scatter_pages([s.reshape(-1) for s in staging], h_cache, bt, n_pages, page_bytes)
+    for l in range(n_layers):
+        assert np.array_equal(d_cache[l].cpu().numpy(), h_cache[l]), l
+    ref = [np.full(floats_each, -7.0, np.float32) for _ in range(n_slots)]
+    if floats_each:
+        oracle.copy_slots(src_h, ref, floats_each)
+    for d, r in zip(dst, ref):
+        assert np.array_equal(d.cpu().numpy().view(np.uint32), r.view(np.uint32))
+
+
+@pytest.mark.parametrize("n_pages", [1, 96, 287])
+def test_restore_request_hybrid_shapes(n_pages):
+    """The one-launch restore of a hybrid request (Section 2.1, Section 5.2): the
+    3 attention layers' pages and the 9 linear layers' 1 MiB states, bit-exact
+    against the oracle's scatter and slot copy."""
+    dev = device()
+    _request_case(dev, HYBRID12.n_full, n_pages, HYBRID12.page_bytes, 600, 9,
+                  HYBRID12.n_heads * HYBRID12.d * HYBRID12.d, seed=n_pages)
+
+
+@pytest.mark.parametrize("case", [dict(n_pages=0), dict(n_layers=0), dict(n_slots=0),
+                                  dict(floats_each=0), dict(floats_each=16 * 4100),
+                                  dict(page_bytes=16 * 37, n_pages=33)])
+def test_restore_request_empty_and_ragged_parts(case):
+    dev = device()
+    a = dict(n_layers=2, n_pages=5, page_bytes=4096, num_blocks=64, n_slots=3,
+             floats_each=4096 * 4)
+    a.update(case)
+    _request_case(dev, a["n_layers"], a["n_pages"], a["page_bytes"], a["num_blocks"],
+                  a["n_slots"], a["floats_each"], seed=11)
+
+
+def test_restore_request_reports_and_skips_bad_units():
+    """An out-of-range block, a NULL state slot and a misaligned state slot are
+    reported and skipped; every other unit is still copied."""
+    dev = device()
+    P, nb, fe = 4096, 8, 16384 * 2 + 4
+    st = torch.arange(3 * P // 4, dtype=torch.int32, device=dev).view(torch.uint8).contiguous()
+    cache = torch.full((nb * P,), POISON, dtype=torch.uint8, device=dev)
+    bt = torch.tensor([2, 9, 5], dtype=torch.int32, device=dev)
+    a = torch.randn(fe, device=dev)
+    b = torch.randn(fe + 4, device=dev)
+    good = torch.zeros(fe, device=dev)
+    nul = torch.zeros(fe, device=dev)
+    mis = torch.zeros(fe + 4, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_restore_request(hs.ptr_array([st], dev), hs.ptr_array([cache], dev), 1, bt, 3, P, nb,
+                          hs.ptr_array([a, 0, b.data_ptr() + 4], dev),
+                          hs.ptr_array([good, nul, mis], dev), 3, fe, err)
+    torch.cuda.synchronize()
+    assert err.item() in (hs.HS_DEVERR_BLOCK_OOB, hs.HS_DEVERR_NULL, hs.HS_DEVERR_MISALIGNED)
+    c = cache.cpu().numpy().reshape(nb, P)
+    s = st.cpu().numpy().reshape(3, P)
+    assert np.array_equal(c[2], s[0]) and np.array_equal(c[5], s[2])
+    assert (np.delete(c, [2, 5], axis=0) == POISON).all()
+    assert torch.equal(good, a)
+    assert not nul.any() and not mis.any()
+    # each kind alone gives its own code
+    for srcs, dsts, table, code in [([a], [good], [2, 9, 5], hs.HS_DEVERR_BLOCK_OOB),
+                                    ([0], [good], [2, 1, 5], hs.HS_DEVERR_NULL),
+                                    ([b.data_ptr() + 4], [mis], [2, 1, 5],
+                                     hs.HS_DEVERR_MISALIGNED)]:
+        err.zero_()
+        hs.hs_restore_request(hs.ptr_array([st], dev), hs.ptr_array([cache], dev), 1,
+                              torch.tensor(table, dtype=torch.int32, device=dev), 3, P, nb,
+                              hs.ptr_array(srcs, dev), hs.ptr_array(dsts, dev), 1, fe, err)
+        torch.cuda.synchronize()
+        assert err.item() == code
+
+
+def test_restore_request_from_pinned_host():
+    """Staging pages and checkpoint slots in pinned host memory, read by the kernel
+    over the C2C link (a restore straight from the host tier)."""
+    dev = device()
+    L, n_pages, P, nb, n_slots, fe = 3, 40, HYBRID12.page_bytes, 200, 9, 16384 * 4
+    staging = [gen_kv_pages(5, l, n_pages, P).reshape(-1) for l in range(L)]
+    h_st = [torch.from_numpy(s).pin_memory() for s in staging]
+    rng = np.random.default_rng(5)
+    src_h = [rng.standard_normal(fe).astype(np.float32) for _ in range(n_slots)]
+    h_src = [torch.from_numpy(x).pin_memory() for x in src_h]
+    bt = gen_block_table(5, 0, n_pages, nb)
+    cache = [torch.full((nb * P,), POISON, dtype=torch.uint8, device=dev) for _ in range(L)]
+    dst = [torch.zeros(fe, device=dev) for _ in range(n_slots)]
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    hs.hs_restore_request(hs.ptr_array(h_st, dev), hs.ptr_array(cache, dev), L,
+                          torch.from_numpy(bt).to(dev), n_pages, P, nb, hs.ptr_array(h_src, dev),
+                          hs.ptr_array(dst, dev), n_slots, fe, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    h_cache = [np.full(nb * P, POISON, np.uint8) for _ in range(L)]
+    oracle.scatter_pages(staging, h_cache, bt, n_pages, P)
+    for l in range(L):
+        assert np.array_equal(cache[l].cpu().numpy(), h_cache[l])
+    for d, r in zip(dst, src_h):
+        assert np.array_equal(d.cpu().numpy().view(np.uint32), r.view(np.uint32))
