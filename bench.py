@@ -153,6 +153,27 @@ class Clocks:
 # the workload on the device
 # ---------------------------------------------------------------------------
 
+def _arena(torch, dev, fields):
+    """One device byte buffer holding typed views [(name, dtype, shape)], each view
+    starting on a 256-byte boundary."""
+    offs, off = [], 0
+    for _, dt, shp in fields:
+        n = 1
+        for x in shp:
+            n *= x
+        offs.append(off)
+        off += -(-(n * torch.empty((), dtype=dt).element_size()) // 256) * 256
+    arena = torch.empty(off, dtype=torch.uint8, device=dev)
+    views = {}
+    for (name, dt, shp), o in zip(fields, offs):
+        n = 1
+        for x in shp:
+            n *= x
+        nb = n * torch.empty((), dtype=dt).element_size()
+        views[name] = arena[o:o + nb].view(dt).view(shp)
+    return arena, views
+
+
 class Hybrid12:
     """Device-resident buffers for the nine-length serial hybrid workload."""
 
@@ -178,28 +199,40 @@ class Hybrid12:
             c, n_pages, tail = hs.hs_align_prefix(L, L, list(range(S.ckpt, L + 1, S.ckpt)), S.page)
             assert tail == TAIL
             self.req.append(dict(L=L, c=c, n_pages=n_pages))
-        # per (seed, request) inputs
+        # per (seed, request) inputs, all of a request's in one contiguous arena (so that
+        # the end-to-end run moves them with one host-to-device copy)
         self.inp = {}
+        tok = (self.nL, self.T, self.nH, self.d)
         for s in range(seeds):
             for r, R in enumerate(self.req):
                 q, k, v, a = torch_gen_linear(100 * s + r, 0, self.nL, self.T, self.nH, self.d, dev)
-                staging = torch.empty((self.nF, max(R["n_pages"], 1) * self.page_bytes),
-                                      dtype=torch.uint8, device=dev)
+                arena, views = _arena(torch, dev, [
+                    ("q", torch.bfloat16, tok), ("k", torch.bfloat16, tok),
+                    ("v", torch.bfloat16, tok), ("a", torch.float32, tok),
+                    ("staging", torch.uint8, (self.nF, max(R["n_pages"], 1) * self.page_bytes)),
+                    ("ck", torch.float32, (self.nL, self.state_floats))])
+                views["q"].copy_(q)
+                views["k"].copy_(k)
+                views["v"].copy_(v)
+                views["a"].copy_(a)
+                del q, k, v, a
+                q, k, v, a, staging, ck = (views[x] for x in ("q", "k", "v", "a", "staging", "ck"))
                 torch_fill_bf16_normal(staging, 1000 * s + r)
-                ck = torch.randn((self.nL, self.state_floats), device=dev,
-                                 generator=torch.Generator(device=dev).manual_seed(7 * s + r)) * 0.5
+                ck.copy_(torch.randn((self.nL, self.state_floats), device=dev,
+                                     generator=torch.Generator(device=dev).manual_seed(7 * s + r)) * 0.5)
                 bt = torch.from_numpy(gen_block_table(s, r, max(R["n_pages"], 1), num_blocks)).to(dev)
                 self.inp[(s, r)] = dict(
-                    q=q, k=k, v=v, a=a, staging=staging, ck=ck, bt=bt,
+                    arena=arena, q=q, k=k, v=v, a=a, staging=staging, ck=ck, bt=bt,
                     staging_ptrs=hs.ptr_array([staging[l] for l in range(self.nF)], dev),
                     ck_ptrs=hs.ptr_array([ck[l] for l in range(self.nL)], dev))
         # per-request outputs (reused across seeds)
         self.out = []
         for r, R in enumerate(self.req):
-            live = torch.empty((self.nL, self.state_floats), device=dev)
-            o = torch.empty((self.nL, self.T, self.nH, self.d), device=dev)
-            emit = torch.empty((self.nL, self.state_floats), device=dev)
-            self.out.append(dict(live=live, o=o, emit=emit,
+            arena, views = _arena(torch, dev, [
+                ("o", torch.float32, tok), ("live", torch.float32, (self.nL, self.state_floats)),
+                ("emit", torch.float32, (self.nL, self.state_floats))])
+            live, o, emit = views["live"], views["o"], views["emit"]
+            self.out.append(dict(arena=arena, live=live, o=o, emit=emit,
                                  live_ptrs=hs.ptr_array([live[l] for l in range(self.nL)], dev),
                                  emit_ptrs=hs.ptr_array([emit[l] for l in range(self.nL)], dev)))
         self.shape = hs.make_shape(self.nL, self.nH, self.d, self.d, self.T, hs.HS_LINATTN_AUTO)
@@ -617,8 +650,11 @@ def e2e_run(wl, steps, warmup):
     h2d = d2h = 0
     for r in range(N_REQ):
         I, O = wl.inp[(0, r)], wl.out[r]
-        hb = {k: I[k].cpu().pin_memory() for k in ("q", "k", "v", "a", "staging", "ck")}
-        ob = {k: torch.empty(O[k].shape, dtype=O[k].dtype).pin_memory() for k in ("o", "live", "emit")}
+        # one pinned buffer per request each way, mirroring the device arenas: every
+        # request's inputs (q, k, v, log-gates, KV staging pages, checkpoint state) arrive
+        # in one copy and its outputs (o, live state, emitted checkpoint) leave in one
+        hb = {"arena": I["arena"].cpu().pin_memory()}
+        ob = {"arena": torch.empty(O["arena"].shape, dtype=torch.uint8).pin_memory()}
         host.append((hb, ob))
         h2d += sum(t.numel() * t.element_size() for t in hb.values())
         d2h += sum(t.numel() * t.element_size() for t in ob.values())
