@@ -503,7 +503,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     }
     if (warp == 0)
         tmem_alloc(sb + OFF_MISC, TMEM_COLS);
-    pdl_wait_and_release();
+    pdl_wait();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
