@@ -56,9 +56,11 @@ using namespace ptx;
 
 constexpr int D = 128;    // d_k = d_v
 constexpr int CH = 64;    // chunk length (absolute grid)
-constexpr int NW = 256;   // worker threads (warps 0..7): operands, state passes, epilogues
-constexpr int NT = NW + 32;  // + one warp whose lane 0 issues every MMA and TMA copy
-constexpr int kIssuer = NW;
+constexpr int NB = 256;   // operand builders (warps 0..7): cumulative gates, Q~, K~, K~^T, V^T
+constexpr int NW = 256;   // state warps (warps 8..15): state passes, masks, epilogues
+constexpr int NT = NB + NW;
+constexpr int kLoader = 0;   // the first builder thread issues every TMA copy
+constexpr int kIssuer = NB;  // the first state thread issues every MMA
 constexpr int kShort = 8; // segments of at most this many tokens run token by token
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kF16Lim = 32768.0f;         // fast-path fp16 operands stay below 2^15
@@ -78,12 +80,13 @@ constexpr uint32_t OFF_SQ = 114688;     // staged q  bf16 [64][128]             
 constexpr uint32_t OFF_SK = 131072;     // staged k                                 16 KiB
 constexpr uint32_t OFF_SV = 147456;     // staged v                                 16 KiB
 constexpr uint32_t OFF_SG = 163840;     // staged log-gates f32 [64][128]           32 KiB
-constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim, one buffer per parity   1 KiB
-constexpr uint32_t OFF_TOT = 197632;    // partial log2-decay totals [4 token quarters][128]  2 KiB
-constexpr uint32_t OFF_RED = 199680;    // per warp [8][8]: max |q|, fast-path flag, max |k|, max |v|, max |S|
-constexpr uint32_t OFF_BAR = 199936;    // 4 mbarriers
-constexpr uint32_t OFF_MISC = 199968;   // TMEM base address, abort flag
-constexpr uint32_t SMEM_BYTES = 200000 + 1024;
+constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim, four slots by chunk number   2 KiB
+constexpr uint32_t OFF_TOT = 198656;    // partial log2-decay totals [4 token quarters][128]  2 KiB
+constexpr uint32_t OFF_RED = 200704;    // per warp [8][8]: builders max |q|, fast-path flag, max |k|,
+                                        //   max |v| (0..3); state warps max |S| (4)
+constexpr uint32_t OFF_BAR = 200960;    // 6 mbarriers
+constexpr uint32_t OFF_MISC = 201024;   // TMEM base address, abort flag, decision, run result
+constexpr uint32_t SMEM_BYTES = 201056 + 1024;
 constexpr uint32_t STAGE_BYTES = 3 * 16384 + 32768;
 
 // tensor memory: D_O alternates between two buffers by chunk parity, placed on
@@ -122,10 +125,31 @@ __device__ __forceinline__ uint32_t t_off(int rows, int row, int col)
                       ((col & 3) << 2));
 }
 
-// barrier among the eight operand warps only (the MMA-issuing warp does not take part)
-__device__ __forceinline__ void bar_workers()
+// barriers among the builder warps (id 1) and among the state warps (id 2)
+__device__ __forceinline__ void bar_builders()
 {
     asm volatile("bar.sync 1, 256;" ::: "memory");
+}
+
+__device__ __forceinline__ void bar_staters()
+{
+    asm volatile("bar.sync 2, 256;" ::: "memory");
+}
+
+// named barrier `id` over 256 threads that also returns the OR of `pred` over them, so
+// every thread of the group takes the same branch after it
+__device__ __forceinline__ bool bar_or(int id, bool pred)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, %2, 256, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)pred), "r"(id)
+        : "memory");
+    return r != 0;
 }
 
 __device__ __forceinline__ float warp_max(float v)
@@ -184,14 +208,14 @@ __device__ __forceinline__ float rna_tf32(float x)
 }
 
 
-// zero the staged rows past a segment of L < 64 tokens (all threads, or the operand
+// zero the staged rows past a segment of L < 64 tokens (all threads, or the builder
 // warps only)
-__device__ __forceinline__ void zero_tail(uint8_t *smem, int L, bool workers_only)
+__device__ __forceinline__ void zero_tail(uint8_t *smem, int L, bool builders_only)
 {
     const int tid = threadIdx.x;
 
     if (L < CH) {
-        const int nthr = workers_only ? NW : NT;
+        const int nthr = builders_only ? NB : NT;
         for (int idx = tid; idx < (CH - L) * 80; idx += nthr) {
             const int row = L + idx / 80, c = idx % 80;
             uint4 *dst;
@@ -205,22 +229,22 @@ __device__ __forceinline__ void zero_tail(uint8_t *smem, int L, bool workers_onl
                 dst = reinterpret_cast<uint4 *>(smem + OFF_SG + row * 512) + (c - 48);
             *dst = make_uint4(0u, 0u, 0u, 0u);
         }
-        if (workers_only)
-            bar_workers();
+        if (builders_only)
+            bar_builders();
         else
             __syncthreads();
     }
 }
 
 
-// ---- fast operands of a staged long segment into set `par`.  Thread (dp, qt) owns key
-// dims 2dp, 2dp+1 for tokens [16 qt, 16 qt + 16): it sums their log2-gates, then runs
-// the cumulative sum again from the earlier quarters' totals (shared memory;
-// 2^{Lam_last} into gam[par]) while it writes
-// Q~ and K~ (token-major, the d-contractions' operands) and K~^T (rows of [A ; K~^T]),
-// fp16, with 4- and 16-byte stores.  Then thread (e, half) packs V^T into TMEM.  Per
-// warp: max |q|, |k|, |v| and whether every operand fits fp16 (for the guard).
-__device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, int par)
+// ---- fast operands of a staged long segment into set `par` (builder warps).  Thread
+// (dp, qt) owns key dims 2dp, 2dp+1 for tokens [16 qt, 16 qt + 16): it sums their
+// log2-gates, then runs the cumulative sum again from the earlier quarters' totals (shared
+// memory; 2^{Lam_last} into gam slot `gslot`) while it writes Q~ and K~ (token-major, the
+// d-contractions' operands) and K~^T (rows of [A ; K~^T]), fp16, with 4- and 16-byte
+// stores.  Then thread (e, half) packs V^T into TMEM.  Per warp: max |q|, |k|, |v| and
+// whether every operand fits fp16 (for the guard).
+__device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, int par, int gslot)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool worker = warp < 8;
@@ -253,7 +277,7 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
         }
         *reinterpret_cast<float2 *>(sTot + qt * D + 2 * dp) = make_float2(r0, r1);
     }
-    bar_workers();
+    bar_builders();
     // the running sums start from the earlier quarters' totals
     float run0 = 0.f, run1 = 0.f;
     {
@@ -269,7 +293,7 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
             t1 += t.y;
         }
         if (qt == 0)
-            *reinterpret_cast<float2 *>(sGam + par * D + 2 * dp) = make_float2(ex2(t0), ex2(t1));
+            *reinterpret_cast<float2 *>(sGam + gslot * D + 2 * dp) = make_float2(ex2(t0), ex2(t1));
     }
     uint8_t *set = smem + par * SET_BYTES;
     const int rowK = par ? 0 : 64;
@@ -341,14 +365,14 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
 }
 
 
-// ---- state pass: decay by gam[gpar] (gpar < 0: none), checkpoint slot, fp16 copy of
-// S^T for the next S^T Q~^T, and the largest |S|
+// ---- state pass (state warps): decay by gam slot gpar (gpar < 0: none), checkpoint slot,
+// fp16 copy of S^T for the next S^T Q~^T, and the largest |S|
 __device__ __forceinline__ void state_pass(uint8_t *smem, uint32_t tmem, int gpar, float *slot, bool copy)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool worker = warp < 8;
+    const bool worker = warp >= 8;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
-    const int colhalf = warp >> 2;
+    const int colhalf = (warp >> 2) & 1;
     const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
     const float *sGam = reinterpret_cast<const float *>(smem + OFF_GAM);
     float *sRed = reinterpret_cast<float *>(smem + OFF_RED);
@@ -402,21 +426,22 @@ __device__ __forceinline__ void state_pass(uint8_t *smem, uint32_t tmem, int gpa
     tmem_wait_st();
     m = warp_max(m);
     if (lane == 0)
-        sRed[warp * 8 + 4] = m;
+        sRed[(warp & 7) * 8 + 4] = m;
 }
 
 
 // ---- the causally masked intra-chunk matrix A (D_A) -> rows rowA.. of set par's [A ; K~^T]
+// (state warps of TMEM lane quarters 0 and 1)
 __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
 {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const bool worker = warp < 8;
+    const bool worker = warp >= 8;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
 
     if (!(worker && (warp & 3) < 2))
         return;
     const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
-    const int jb = (warp >> 2) * 32;            // this warp's 32 key columns
+    const int jb = ((warp >> 2) & 1) * 32;      // this warp's 32 key columns
     const int rowA = par ? 128 : 0;
     float r[32];
     tmem_ld32(tmem + lrow + TM_A + jb, r);
@@ -436,13 +461,14 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
 }
 
 
-// ---- output epilogue of a processed segment: D_O buffer `par` -> o (lane e, 32 rows)
+// ---- output epilogue of a processed segment (state warps): D_O buffer `par` -> o (lane e,
+// 32 rows)
 __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t tstride, int L, int par)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool worker = warp < 8;
+    const bool worker = warp >= 8;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
-    const int colhalf = warp >> 2;
+    const int colhalf = (warp >> 2) & 1;
     const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
 
     if (!worker)
@@ -478,9 +504,14 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     float *sTot = reinterpret_cast<float *>(smem + OFF_TOT);
     float *sGam = reinterpret_cast<float *>(smem + OFF_GAM);
     float *sRed = reinterpret_cast<float *>(smem + OFF_RED);
+    // [0] TMEM base, [1] abort flag, [2] decision on the latest built segment (1 = fast),
+    // [3] run result (1 = the segment at [4..5] needs the exact path), [4..5] position
+    // where the run stopped, [6..7] its local token index
     volatile uint32_t *sMisc = reinterpret_cast<volatile uint32_t *>(smem + OFF_MISC);
+    volatile int64_t *sRun = reinterpret_cast<volatile int64_t *>(smem + OFF_MISC + 16);
     const uint32_t bar_tma = sb + OFF_BAR, bar_a = sb + OFF_BAR + 8, bar_o = sb + OFF_BAR + 16,
-                   bar_s = sb + OFF_BAR + 24;
+                   bar_s = sb + OFF_BAR + 24, bar_built = sb + OFF_BAR + 32,
+                   bar_go = sb + OFF_BAR + 40;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int b = blockIdx.x / p.n_heads;
@@ -498,6 +529,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         mbar_init(bar_a, 1);
         mbar_init(bar_o, 1);
         mbar_init(bar_s, 1);
+        mbar_init(bar_built, 1);
+        mbar_init(bar_go, 1);
         fence_mbar_init();
         sMisc[1] = 0;   // abort flag
     }
@@ -508,17 +541,20 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = sMisc[0];
-    const bool worker = warp < 8;
+    const bool builder = warp < 8;
+    const bool worker = !builder;                              // a state warp
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
-    const int colhalf = warp >> 2;
+    const int colhalf = (warp >> 2) & 1;
     const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
-    // operand-building map: worker owns key dim d = e_own for tokens [32*th, 32*th+32)
+    // exact operand map: state thread owns key dim d = e_own for tokens [32*th, 32*th+32)
     const int d = e_own;
     const int th = colhalf;
 
-    // issuer bookkeeping (lane 0 of warp 8) of copies issued, for the abort path
+    // bookkeeping of the loader (copies issued, one still in flight) and of the issuer,
+    // for the waits and the abort path; every mbarrier is waited on by one thread only
     uint32_t n_tma = 0;
-    uint32_t ph_tma = 0, ph_a = 0, ph_o = 0, ph_s = 0;
+    bool tma_pending = false;
+    uint32_t ph_tma = 0, ph_a = 0, ph_o = 0, ph_s = 0, ph_built = 0, ph_go = 0;
     bool aborted = false;
 
     // L2 prefetch of the 64 tokens from local position t (if any are this problem's)
@@ -532,8 +568,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tma_prefetch_2d(&maps.v, x, y);
         tma_prefetch_2d(&maps.g, x, y);
     };
-    // staged inputs of the segment at local position tok_local; segments after the
-    // first start on the 64-token grid, so the segment kPrefetch ahead starts at
+    // (loader) staged inputs of the segment at local position tok_local; segments after
+    // the first start on the 64-token grid, so the segment kPrefetch ahead starts at
     // tok_local + 64 * kPrefetch and is requested into L2 now
     auto issue_tma = [&](int64_t tok_local) {
         const int32_t y = (int32_t)((int64_t)p.row0[b] + tok_local);
@@ -544,49 +580,64 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tma_load_2d(sb + OFF_SV, &maps.v, x, y, bar_tma);
         tma_load_2d(sb + OFF_SG, &maps.g, x, y, bar_tma);
         ++n_tma;
+        tma_pending = true;
         if (tok_local > 0)
             prefetch(tok_local + (int64_t)CH * kPrefetch);
     };
-    // the issuer waits on an mbarrier, then everyone meets; false if a wait ran out
-    auto wait_all = [&](uint32_t bar, uint32_t &ph) -> bool {
-        if (tid == kIssuer && !mbar_wait_bounded(bar, ph, kTimeoutNs))
+    // one thread (`who`) waits on an mbarrier; false (for every thread) if that wait ran
+    // out or another thread raised the abort flag.  CTA-wide, or within the builder (id 1)
+    // or state (id 2) warps; the barrier's OR reduction makes the answer uniform.
+    auto wait_all = [&](int who, uint32_t bar, uint32_t &ph) -> bool {
+        bool bad = false;
+        if (tid == who)
+            bad = !mbar_wait_bounded(bar, ph, kTimeoutNs);
+        if (bad)
             sMisc[1] = 1;
-        __syncthreads();
+        ph ^= 1;
+        const bool stop = __syncthreads_or(bad || sMisc[1] != 0) != 0;
         tc_fence_after();
-        ph ^= 1;
-        if (sMisc[1]) {
+        if (stop)
             aborted = true;
-            return false;
-        }
-        return true;
+        return !stop;
     };
-    auto wait_tma = [&]() -> bool { return wait_all(bar_tma, ph_tma); };
-    // one operand thread waits, then the operand warps meet; the issuer only follows the
-    // phase.  A timeout is seen by everyone at the next sync_all.
-    auto wait_w = [&](uint32_t bar, uint32_t &ph) {
-        if (tid == 0 && !mbar_wait_bounded(bar, ph, kTimeoutNs))
+    auto wait_tma = [&]() -> bool {
+        tma_pending = false;
+        return wait_all(kLoader, bar_tma, ph_tma);
+    };
+    auto wait_group = [&](int id, int who, uint32_t bar, uint32_t &ph) -> bool {
+        bool bad = false;
+        if (tid == who)
+            bad = !mbar_wait_bounded(bar, ph, kTimeoutNs);
+        if (bad)
             sMisc[1] = 1;
-        if (worker) {
-            bar_workers();
-            tc_fence_after();
-        }
         ph ^= 1;
+        const bool stop = bar_or(id, bad || sMisc[1] != 0);
+        tc_fence_after();
+        if (stop)
+            aborted = true;
+        return !stop;
+    };
+    // a group barrier that also reports the abort flag, uniformly
+    auto sync_group = [&](int id) -> bool {
+        const bool stop = bar_or(id, sMisc[1] != 0);
+        if (stop)
+            aborted = true;
+        return !stop;
     };
     auto sync_all = [&]() -> bool {
-        __syncthreads();
-        if (sMisc[1]) {
+        const bool stop = __syncthreads_or(sMisc[1] != 0) != 0;
+        if (stop)
             aborted = true;
-            return false;
-        }
-        return true;
+        return !stop;
     };
     auto seg_len = [&](int64_t at) -> int { return (int)(min(end, (at / CH + 1) * CH) - at); };
+    auto is_long = [&](int64_t at) -> bool { return at < end && seg_len(at) > kShort; };
     auto ckpt_slot = [&](int64_t seg_end) -> float * {
         if (!(C > 0 && seg_end % C == 0 && p.ckpt_slots != nullptr))
             return nullptr;
         float *slot = p.ckpt_slots[p.ck_base[b] + (seg_end / C - pos0 / C - 1)];
         if (slot == nullptr || (reinterpret_cast<uintptr_t>(slot) & 15u) != 0) {
-            if (tid == 0)
+            if (tid == kIssuer)
                 report(p.d_err, slot == nullptr ? HS_DEVERR_NULL : HS_DEVERR_MISALIGNED);
             return nullptr;
         }
@@ -601,10 +652,16 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         return m;
     };
 
-    if (tid == kIssuer)
+    if (tid == kLoader) {
         issue_tma(0);
+        // the first kPrefetch segments after the first one
+        const int64_t t1 = min(end, (pos0 / CH + 1) * CH) - pos0;
+        for (int j = 0; j < kPrefetch; ++j)
+            prefetch(t1 + (int64_t)CH * j);
+    }
 
-    // incoming state -> TMEM, transposed: S^T[e][d] = state[d][e]; its largest magnitude
+    // incoming state -> TMEM (state warps), transposed: S^T[e][d] = state[d][e]; its
+    // largest magnitude.  The builders meanwhile stage and build the first segment.
     float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
     if (worker) {
         float r[32];
@@ -622,17 +679,10 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tmem_wait_st();
         m = warp_max(m);
         if (lane == 0)
-            sRed[warp * 8 + 4] = m;
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (tid == kIssuer) {
-        // the first kPrefetch segments after the first one, once the state is in: the
-        // state and the first segment are not queued behind them
-        const int64_t t1 = min(end, (pos0 / CH + 1) * CH) - pos0;
-        for (int j = 0; j < kPrefetch; ++j)
-            prefetch(t1 + (int64_t)CH * j);
+            sRed[(warp & 7) * 8 + 4] = m;
+        tc_fence_before();
+        bar_staters();
+        tc_fence_after();
     }
 
     // ---- a short segment (<= kShort tokens, staged inputs already waited for, no decay
@@ -674,12 +724,12 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             m = warp_max(m);
             if (lane == 0)
-                sRed[warp * 8 + 4] = m;
+                sRed[(warp & 7) * 8 + 4] = m;
             tmem_wait_st();
         }
         fence_proxy_async_smem();
         __syncthreads();
-        if (tid == kIssuer && seg_end < end)
+        if (tid == kLoader && seg_end < end)
             issue_tma(tok_s + L);
         float *ob = p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D;
         for (int idx = tid; idx < L * D; idx += NT) {
@@ -695,15 +745,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         tc_fence_after();
     };
 
-
-
-
-
-
-    // the guard of a built fast segment (after the barrier that follows build_fast): log-gates
-    // <= 0, and every fp16 operand (Q~, K~, V, A, the fp16 copy of the state it starts
-    // from) below 2^15 in magnitude
-    float mk_cur = 0.f, mv_cur = 0.f;   // maxima |k|, |v| of the pending fast segment
+    // the guard of a built fast segment (state warps, after the wait for the builders): log-gates
+    // <= 0, and every fp16 operand (Q~, K~, V, A, the fp16 copy of the state it starts from)
+    // below 2^15 in magnitude
     float mk_new = 0.f, mv_new = 0.f;
     auto guard = [&](float s_bound) -> bool {
         float mq = 0.f, mk = 0.f, mv = 0.f;
@@ -722,7 +766,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
 
     // ---- one exact segment, from staged inputs, no decay pending and no MMA in flight;
     // leaves the final state in TMEM, writes its outputs and checkpoint
-    auto exact_segment = [&](int64_t tok_s, int L, int par, int64_t seg_end) -> bool {
+    auto exact_segment = [&](int64_t tok_s, int L, int par, int gslot, int64_t seg_end) -> bool {
         // cumulative log2-gates: key dim d over 32 tokens per thread, halves joined through
         // shared memory; 2^{Lam_last} into gam[par]
         float lam[32];
@@ -747,7 +791,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     for (int x = 0; x < 32; ++x)
                         lam[x] = tot0 + lam[x];
                 } else {
-                    sGam[par * D + d] = ex2(last);
+                    sGam[gslot * D + d] = ex2(last);
                 }
             }
         }
@@ -815,9 +859,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             tc_commit(bar_o);
         }
-        if (!wait_all(bar_o, ph_o))
+        if (!wait_all(kIssuer, bar_o, ph_o))
             return false;
-        state_pass(smem, tmem, par, nullptr, false);          // S <- diag(2^{Lam_last}) S
+        state_pass(smem, tmem, gslot, nullptr, false);          // S <- diag(2^{Lam_last}) S
         tc_fence_before();
         __syncthreads();
         if (tid == kIssuer) {
@@ -830,7 +874,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             tc_commit(bar_s);
         }
-        if (!wait_all(bar_s, ph_s))
+        if (!wait_all(kIssuer, bar_s, ph_s))
             return false;
         state_pass(smem, tmem, -1, ckpt_slot(seg_end), false);   // checkpoint and |S| of the final state
         out_epilogue(tmem, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride, L, par);
@@ -840,70 +884,77 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         return true;
     };
 
-    int64_t pos = pos0, tok = 0;
-    // leading short segment
-    if (seg_len(pos) <= kShort) {
-        if (!wait_tma())
-            goto finish;
-        short_segment(tok, seg_len(pos), pos + seg_len(pos));
-        tok += seg_len(pos);
-        pos += seg_len(pos);
-    }
-
-    // ---- long segments: fast ones pipelined two deep, exact ones one at a time
-    {
-        const auto out_of = [&](int64_t t) {
-            return p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D;
-        };
+    // ---- a run of long segments on the fast path, the two groups of warps in a pipeline:
+    // the builders stage and build segment k+1 while the state warps finish segment k.
+    // Handoffs (each mbarrier has one waiting thread and one arriving party):
+    //   bar_built: builders -> state warps, segment k built (operands, V^T, guard maxima)
+    //   bar_go:    state warps -> builders, the decision on segment k is made (sMisc[2]);
+    //              when it is fast, it also means the operand set of segment k+1 is free
+    //              (the products of segment k-1 are complete)
+    // A run ends after the last long segment or before a segment the guard sends to the
+    // exact path; the groups then meet CTA-wide.  No MMA is in flight at either end.
+    auto outp = [&](int64_t t) { return p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D; };
+    int kseq = 0;   // long segments of the current run so far (slot of 2^{Lam_last}: kseq mod 4)
+    auto builder_run = [&](int64_t rpos, int64_t rtok) {
         int par = 0;
-        bool have_prep = false, prep_fast = false, qk_issued = false;
-        bool pend = false;
-        int pend_par = 0, pend_L = 0;
+        while (true) {
+            const int L = seg_len(rpos);
+            if (!wait_group(1, kLoader, bar_tma, ph_tma))
+                return;
+            tma_pending = false;
+            build_fast(smem, tmem, L, par, kseq & 3);
+            fence_proxy_async_smem();
+            tc_fence_before();
+            if (!sync_group(1))
+                return;
+            const bool next_long = is_long(rpos + L);
+            if (tid == kLoader) {
+                mbar_arrive(bar_built);
+                // the staged rows are consumed: stage the next segment (long or short) now;
+                // an exact decision on this one reloads it
+                if (rpos + L < end)
+                    issue_tma(rtok + L);
+            }
+            if (!wait_group(1, kLoader, bar_go, ph_go))
+                return;
+            if (sMisc[2] == 0 || !next_long)
+                return;
+            rpos += L;
+            rtok += L;
+            par ^= 1;
+            ++kseq;
+        }
+    };
+    auto state_run = [&](int64_t rpos, int64_t rtok) {
+        int par = 0;
+        bool pend = false, stop_exact = false;
+        int pend_par = 0, pend_L = 0, pend_g = 0;
         int64_t pend_tok = 0, pend_end = 0;
-        while (pos < end && seg_len(pos) > kShort) {
-            const int L = seg_len(pos);
-            const int64_t seg_end = pos + L;
-            const bool has_next = seg_end < end;
-            if (!have_prep) {
-                wait_w(bar_tma, ph_tma);
-                build_fast(smem, tmem, L, par);
-                fence_proxy_async_smem();
-                tc_fence_before();
-                if (!sync_all())
-                    break;
-                prep_fast = guard(state_max());
-                if (prep_fast && tid == kIssuer && has_next)
-                    issue_tma(tok + L);
-            }
-            if (!prep_fast) {
-                if (pend) {
-                    if (!wait_all(bar_o, ph_o))
-                        break;
-                    state_pass(smem, tmem, pend_par, ckpt_slot(pend_end), false);
-                    out_epilogue(tmem, out_of(pend_tok), tstride, pend_L, pend_par);
-                    tc_fence_before();
-                    __syncthreads();
-                    tc_fence_after();
-                    pend = false;
-                }
-                if (!exact_segment(tok, L, par, seg_end))
-                    break;
-                if (tid == kIssuer && has_next)
-                    issue_tma(tok + L);
-                pos = seg_end;
-                tok += L;
-                have_prep = false;
-                qk_issued = false;
-                continue;
-            }
+        float mk_cur = 0.f, mv_cur = 0.f;
+        if (!wait_group(2, kIssuer, bar_built, ph_built))
+            return;
+        bool fast = guard(state_max());
+        if (tid == kIssuer) {
+            sMisc[2] = fast ? 1u : 0u;
+            if (!fast)
+                mbar_arrive(bar_go);
+        }
+        stop_exact = !fast;
+        bool qk_issued = false;
+        while (fast) {
+            const int L = seg_len(rpos);
+            const int64_t seg_end = rpos + L;
             mk_cur = mk_new;
             mv_cur = mv_new;
-            if (pend)
-                wait_w(bar_o, ph_o);
-            state_pass(smem, tmem, pend ? pend_par : -1, pend ? ckpt_slot(pend_end) : nullptr, true);
+            if (pend && !wait_group(2, kIssuer, bar_o, ph_o))
+                return;
+            // the products of the previous segment are complete: its operand set is free
+            if (tid == kIssuer)
+                mbar_arrive(bar_go);
+            state_pass(smem, tmem, pend ? pend_g : -1, pend ? ckpt_slot(pend_end) : nullptr, true);
             tc_fence_before();
-            if (!sync_all())
-                break;
+            if (!sync_group(2))
+                return;
             const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
             if (tid == kIssuer) {
                 tc_fence_after();
@@ -924,29 +975,14 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 tc_commit(bar_a);
             }
             if (pend)
-                out_epilogue(tmem, out_of(pend_tok), tstride, pend_L, pend_par);
-            pend = false;
-            const bool next_long = has_next && seg_len(seg_end) > kShort;
-            bool next_fast = false;
-            if (next_long) {
-                const int L1 = seg_len(seg_end);
-                wait_w(bar_tma, ph_tma);
-                build_fast(smem, tmem, L1, par ^ 1);
-                fence_proxy_async_smem();
-                tc_fence_before();
-                if (!sync_all())
-                    break;
-                next_fast = guard(state_max() + 64.0f * mk_cur * mv_cur);
-                if (next_fast && tid == kIssuer && seg_end + L1 < end)
-                    issue_tma(tok + L + L1);
-            }
-            if (!wait_all(bar_a, ph_a))
-                break;
+                out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par);
+            if (!wait_group(2, kIssuer, bar_a, ph_a))
+                return;
             a_build(smem, tmem, par);
             fence_proxy_async_smem();
             tc_fence_before();
-            if (!sync_all())
-                break;
+            if (!sync_group(2))
+                return;
             if (tid == kIssuer) {
                 tc_fence_after();
                 const uint32_t vt = tmem + TM_V + 32 * par;
@@ -955,8 +991,29 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     mma_f16_ts(tmem + (par ? TM_S : TM_O0), vt + kk * 8,
                                sdesc_sw128(setb + S_B2H + kk * 32, 16, 1024), IDF_N192, 1);
                 tc_commit(bar_o);
-                if (next_fast) {
-                    const uint32_t nsetb = sb + (uint32_t)(par ^ 1) * SET_BYTES;
+            }
+            pend = true;
+            pend_par = par;
+            pend_tok = rtok;
+            pend_L = L;
+            pend_end = seg_end;
+            pend_g = kseq & 3;
+            rpos = seg_end;
+            rtok += L;
+            par ^= 1;
+            ++kseq;
+            if (!is_long(rpos))
+                break;
+            // the builders' next segment, and the decision on it
+            if (!wait_group(2, kIssuer, bar_built, ph_built))
+                return;
+            fast = guard(state_max() + 64.0f * mk_cur * mv_cur);
+            if (tid == kIssuer) {
+                sMisc[2] = fast ? 1u : 0u;
+                if (!fast) {
+                    mbar_arrive(bar_go);
+                } else {
+                    const uint32_t nsetb = sb + (uint32_t)par * SET_BYTES;
 #pragma unroll 1
                     for (int kk = 0; kk < D / 16; ++kk) {
                         const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
@@ -965,40 +1022,70 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     }
                 }
             }
-            qk_issued = next_fast;
-            pend = true;
-            pend_par = par;
-            pend_tok = tok;
-            pend_L = L;
-            pend_end = seg_end;
-            pos = seg_end;
-            tok += L;
-            par ^= 1;
-            have_prep = next_long;
-            prep_fast = next_fast;
+            qk_issued = fast;
+            stop_exact = !fast;
         }
-        if (aborted)
-            goto finish;
         if (pend) {
-            if (!wait_all(bar_o, ph_o))
-                goto finish;
-            state_pass(smem, tmem, pend_par, ckpt_slot(pend_end), false);
-            out_epilogue(tmem, out_of(pend_tok), tstride, pend_L, pend_par);
+            if (!wait_group(2, kIssuer, bar_o, ph_o))
+                return;
+            state_pass(smem, tmem, pend_g, ckpt_slot(pend_end), false);
+            out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par);
             tc_fence_before();
-            __syncthreads();
-            tc_fence_after();
+            if (!sync_group(2))
+                return;
+        }
+        if (tid == kIssuer) {
+            sMisc[3] = stop_exact ? 1u : 0u;
+            sRun[0] = rpos;
+            sRun[1] = rtok;
+        }
+    };
+
+    int64_t pos = pos0, tok = 0;
+    while (pos < end) {
+        const int L = seg_len(pos);
+        if (L <= kShort) {
+            // a leading or trailing short segment (its inputs are staged or in flight)
+            if (!wait_tma())
+                break;
+            short_segment(tok, L, pos + L);
+            pos += L;
+            tok += L;
+            continue;
+        }
+        if (builder)
+            builder_run(pos, tok);
+        else
+            state_run(pos, tok);
+        if (!sync_all())
+            break;
+        tc_fence_after();
+        const bool exact = sMisc[3] != 0;
+        pos = sRun[0];
+        tok = sRun[1];
+        kseq = 0;
+        if (exact) {
+            // the segment at pos takes the exact path: restage its inputs (the copy of the
+            // next segment may be in flight), then every thread runs it
+            const int Lx = seg_len(pos);
+            if (tid == kLoader) {
+                if (tma_pending && !mbar_wait_bounded(bar_tma, ph_tma, kTimeoutNs))
+                    sMisc[1] = 1;
+                if (tma_pending)
+                    ph_tma ^= 1;
+                issue_tma(tok);
+            }
+            if (!wait_tma())
+                break;
+            if (!exact_segment(tok, Lx, 0, 0, pos + Lx))
+                break;
+            pos += Lx;
+            tok += Lx;
+            if (tid == kLoader && pos < end)
+                issue_tma(tok);
         }
     }
 
-    // trailing short segment (its inputs were requested by the previous segment)
-    if (pos < end) {
-        if (!wait_tma())
-            goto finish;
-        short_segment(tok, seg_len(pos), pos + seg_len(pos));
-        pos += seg_len(pos);
-    }
-
-finish:
     if (!aborted) {
         if (worker) {
             // final state back to global memory, row = key dim
@@ -1013,13 +1100,17 @@ finish:
                     st_g[(int64_t)(d0 + x) * D + e_own] = r[x];
             }
         }
-    } else if (tid == kIssuer) {
-        report(p.d_err, HS_DEVERR_TIMEOUT);
+    } else {
         // let this CTA's own copies and MMAs drain (bounded) before its memory goes away
-        if (n_tma > 0)
-            mbar_wait_bounded(bar_tma, (n_tma - 1) & 1, kTimeoutNs);
-        tc_commit(bar_s);
-        mbar_wait_bounded(bar_s, ph_s, kTimeoutNs);
+        if (tid == kLoader) {
+            report(p.d_err, HS_DEVERR_TIMEOUT);
+            if (n_tma > 0)
+                mbar_wait_bounded(bar_tma, (n_tma - 1) & 1, kTimeoutNs);
+        }
+        if (tid == kIssuer) {
+            tc_commit(bar_s);
+            mbar_wait_bounded(bar_s, ph_s, kTimeoutNs);
+        }
     }
     tc_fence_before();
     __syncthreads();
