@@ -84,7 +84,7 @@ constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim, four slots 
 constexpr uint32_t OFF_TOT = 198656;    // partial log2-decay totals [4 token quarters][128]  2 KiB
 constexpr uint32_t OFF_RED = 200704;    // per warp [8][8]: builders max |q|, fast-path flag, max |k|,
                                         //   max |v| (0..3); state warps max |S| (4)
-constexpr uint32_t OFF_BAR = 200960;    // 6 mbarriers
+constexpr uint32_t OFF_BAR = 200960;    // 8 mbarriers
 constexpr uint32_t OFF_MISC = 201024;   // TMEM base address, abort flag, decision, run result
 constexpr uint32_t SMEM_BYTES = 201056 + 1024;
 constexpr uint32_t STAGE_BYTES = 3 * 16384 + 32768;
@@ -98,8 +98,9 @@ constexpr uint32_t TM_O0 = 0;           // D_O of even chunks (lane e, col i), 6
 constexpr uint32_t TM_S = 64;           // S^T  float32, 128 lanes x 128 cols
 constexpr uint32_t TM_O1 = 192;         // D_O of odd chunks
 constexpr uint32_t TM_SH = 256;         // S^T fp16 copy, two key dims per column      64 cols
-constexpr uint32_t TM_A = 320;          // D_A  128 lanes x 64 cols (lanes 0..63 used)
+constexpr uint32_t TM_A0 = 320;         // D_A of even segments, 128 lanes x 64 cols (lanes 0..63 used)
 constexpr uint32_t TM_V = 384;          // V^T: fast, fp16 pairs 2 x 32 cols; exact, f32 64 cols
+constexpr uint32_t TM_A1 = 448;         // D_A of odd segments
 
 constexpr uint32_t IDF_N64 = idesc_f16(128, 64);
 constexpr uint32_t IDF_N192 = idesc_f16(128, 192);
@@ -444,7 +445,7 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
     const int jb = ((warp >> 2) & 1) * 32;      // this warp's 32 key columns
     const int rowA = par ? 128 : 0;
     float r[32];
-    tmem_ld32(tmem + lrow + TM_A + jb, r);
+    tmem_ld32(tmem + lrow + (par ? TM_A1 : TM_A0) + jb, r);
     tmem_wait_ld();
     uint8_t *set = smem + par * SET_BYTES;
 #pragma unroll
@@ -511,7 +512,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     volatile int64_t *sRun = reinterpret_cast<volatile int64_t *>(smem + OFF_MISC + 16);
     const uint32_t bar_tma = sb + OFF_BAR, bar_a = sb + OFF_BAR + 8, bar_o = sb + OFF_BAR + 16,
                    bar_s = sb + OFF_BAR + 24, bar_built = sb + OFF_BAR + 32,
-                   bar_go = sb + OFF_BAR + 40;
+                   bar_go = sb + OFF_BAR + 40, bar_ld = sb + OFF_BAR + 48,
+                   bar_a1 = sb + OFF_BAR + 56;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int b = blockIdx.x / p.n_heads;
@@ -531,11 +533,23 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         mbar_init(bar_s, 1);
         mbar_init(bar_built, 1);
         mbar_init(bar_go, 1);
+        mbar_init(bar_ld, 1);
+        mbar_init(bar_a1, 1);
         fence_mbar_init();
         sMisc[1] = 0;   // abort flag
     }
     if (warp == 0)
         tmem_alloc(sb + OFF_MISC, TMEM_COLS);
+    if (tid == kLoader) {
+        // the first segment's inputs into L2 while the previous kernel finishes: a
+        // prefetch moves no data into this SM, and L2 holds the only copy any later write
+        // updates, so it is safe even if that kernel writes those inputs
+        const int32_t y = (int32_t)p.row0[b];
+        tma_prefetch_2d(&maps.q, h * D, y);
+        tma_prefetch_2d(&maps.k, h * D, y);
+        tma_prefetch_2d(&maps.v, h * D, y);
+        tma_prefetch_2d(&maps.g, h * D, y);
+    }
     pdl_wait();
     tc_fence_before();
     __syncthreads();
@@ -554,7 +568,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // for the waits and the abort path; every mbarrier is waited on by one thread only
     uint32_t n_tma = 0;
     bool tma_pending = false;
-    uint32_t ph_tma = 0, ph_a = 0, ph_o = 0, ph_s = 0, ph_built = 0, ph_go = 0;
+    uint32_t ph_tma = 0, ph_o = 0, ph_s = 0, ph_built = 0, ph_go = 0;
+    uint32_t ph_a0 = 0, ph_a1 = 0;   // D_A products of even / odd segments (bar_a, bar_a1)
     bool aborted = false;
 
     // L2 prefetch of the 64 tokens from local position t (if any are this problem's)
@@ -652,13 +667,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         return m;
     };
 
-    if (tid == kLoader) {
+    if (tid == kLoader)
         issue_tma(0);
-        // the first kPrefetch segments after the first one
-        const int64_t t1 = min(end, (pos0 / CH + 1) * CH) - pos0;
-        for (int j = 0; j < kPrefetch; ++j)
-            prefetch(t1 + (int64_t)CH * j);
-    }
+    bool prefetched = false;   // (loader) the segments after the first requested into L2
 
     // incoming state -> TMEM (state warps), transposed: S^T[e][d] = state[d][e]; its
     // largest magnitude.  The builders meanwhile stage and build the first segment.
@@ -767,55 +778,58 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // ---- one exact segment, from staged inputs, no decay pending and no MMA in flight;
     // leaves the final state in TMEM, writes its outputs and checkpoint
     auto exact_segment = [&](int64_t tok_s, int L, int par, int gslot, int64_t seg_end) -> bool {
-        // cumulative log2-gates: key dim d over 32 tokens per thread, halves joined through
-        // shared memory; 2^{Lam_last} into gam[par]
-        float lam[32];
-        float last = 0.f;
+        // cumulative log2-gates: key dim d over 32 tokens per thread (token-major into
+        // X_LAM, the elementwise A reads them there), halves joined through shared memory;
+        // 2^{Lam_last} into gam slot gslot
+        float *sLam = reinterpret_cast<float *>(smem + X_LAM);
+        float last = 0.f, tot0 = 0.f;
         zero_tail(smem, L, false);
         {
             float run = 0.f;
             if (worker) {
-#pragma unroll
+#pragma unroll 8
                 for (int x = 0; x < 32; ++x) {
                     run = fmaf(sG[(32 * th + x) * D + d], kLog2e, run);
-                    lam[x] = run;
+                    sLam[(32 * th + x) * D + d] = run;
                 }
                 sTot[th * D + d] = run;
             }
             __syncthreads();
             if (worker) {
-                const float tot0 = sTot[d];
+                tot0 = sTot[d];
                 last = tot0 + sTot[D + d];   // Lam_last of key dim d
-                if (th) {
-#pragma unroll
-                    for (int x = 0; x < 32; ++x)
-                        lam[x] = tot0 + lam[x];
-                } else {
+                if (!th)
                     sGam[gslot * D + d] = ex2(last);
-                }
             }
         }
         if (worker) {
             // Q~ = q 2^{Lam} (tf32), K^^T = k 2^{Lam_last - Lam} (tf32, rows 64.. of X_B2),
-            // Lam token-major for the elementwise A, V^T float32 into TMEM
-            float vtr[32];
+            // V^T float32 into TMEM, 16 tokens at a time
+#pragma unroll 1
+            for (int hh = 0; hh < 2; ++hh) {
+                uint32_t vtr[16];
 #pragma unroll
-            for (int g = 0; g < 8; ++g) {
-                float4 w;
-                float *wv = &w.x;
+                for (int g = 0; g < 4; ++g) {
+                    float4 w;
+                    float *wv = &w.x;
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    const int x = 4 * g + u;
-                    const int i = 32 * th + x;
-                    *reinterpret_cast<float *>(smem + X_QT + t_off(64, i, d)) =
-                        rna_tf32(bf16f(sQ[i * D + d]) * ex2(lam[x]));
-                    wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam[x]));
-                    reinterpret_cast<float *>(smem + X_LAM)[i * D + d] = lam[x];
-                    vtr[x] = bf16f(sV[i * D + d]);
+                    for (int u = 0; u < 4; ++u) {
+                        const int x = 16 * hh + 4 * g + u;
+                        const int i = 32 * th + x;
+                        float lam = sLam[i * D + d];
+                        if (th) {
+                            lam = tot0 + lam;
+                            sLam[i * D + d] = lam;
+                        }
+                        *reinterpret_cast<float *>(smem + X_QT + t_off(64, i, d)) =
+                            rna_tf32(bf16f(sQ[i * D + d]) * ex2(lam));
+                        wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam));
+                        vtr[4 * g + u] = __float_as_uint(bf16f(sV[i * D + d]));
+                    }
+                    *reinterpret_cast<float4 *>(smem + X_B2 + t_off(192, 64 + d, 32 * th + 16 * hh + 4 * g)) = w;
                 }
-                *reinterpret_cast<float4 *>(smem + X_B2 + t_off(192, 64 + d, 32 * th + 4 * g)) = w;
+                tmem_st16(tmem + lrow + TM_V + 32 * th + 16 * hh, vtr);
             }
-            tmem_st32(tmem + lrow + TM_V + 32 * th, vtr);
             tmem_wait_st();
         }
         fence_proxy_async_smem();
@@ -902,6 +916,13 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             if (!wait_group(1, kLoader, bar_tma, ph_tma))
                 return;
             tma_pending = false;
+            if (tid == kLoader && !prefetched) {
+                // once the first segment has landed (the state and the first segment are
+                // not queued behind these): the next kPrefetch segments into L2
+                prefetched = true;
+                for (int j = 1; j <= kPrefetch; ++j)
+                    prefetch(rtok + L + (int64_t)CH * (j - 1));
+            }
             build_fast(smem, tmem, L, par, kseq & 3);
             fence_proxy_async_smem();
             tc_fence_before();
@@ -909,6 +930,17 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 return;
             const bool next_long = is_long(rpos + L);
             if (tid == kLoader) {
+                // D_A = Q~ K~^T of this segment, into its own buffer (the state warps wait on
+                // bar_a / bar_a1 by parity before they read it)
+                tc_fence_after();
+                const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
+#pragma unroll 1
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
+                    mma_f16_ss(tmem + (par ? TM_A1 : TM_A0), sdesc_sw128(setb + S_QH + koff, 16, 1024),
+                               sdesc_sw128(setb + S_KH + koff, 16, 1024), IDF_N64, kk > 0);
+                }
+                tc_commit(par ? bar_a1 : bar_a);
                 mbar_arrive(bar_built);
                 // the staged rows are consumed: stage the next segment (long or short) now;
                 // an exact decision on this one reloads it
@@ -940,7 +972,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 mbar_arrive(bar_go);
         }
         stop_exact = !fast;
-        bool qk_issued = false;
+        // a segment sent to the exact path: its (unused) D_A product is drained first
+        if (!fast && !wait_group(2, kIssuer, bar_a, ph_a0))
+            return;
         while (fast) {
             const int L = seg_len(rpos);
             const int64_t seg_end = rpos + L;
@@ -957,26 +991,19 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 return;
             const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
             if (tid == kIssuer) {
+                // D_O = S^T Q~^T (the N = 192 product below accumulates onto it in order)
                 tc_fence_after();
-                if (!qk_issued) {
-#pragma unroll 1
-                    for (int kk = 0; kk < D / 16; ++kk) {
-                        const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
-                        mma_f16_ss(tmem + TM_A, sdesc_sw128(setb + S_QH + koff, 16, 1024),
-                                   sdesc_sw128(setb + S_KH + koff, 16, 1024), IDF_N64, kk > 0);
-                    }
-                }
 #pragma unroll 1
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
                     mma_f16_ts(tmem + (par ? TM_O1 : TM_O0), tmem + TM_SH + kk * 8,
                                sdesc_sw128(setb + S_QH + koff, 16, 1024), IDF_N64, kk > 0);
                 }
-                tc_commit(bar_a);
             }
             if (pend)
                 out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par);
-            if (!wait_group(2, kIssuer, bar_a, ph_a))
+            // D_A of this segment (issued by the builders' loader)
+            if (!(par ? wait_group(2, kIssuer, bar_a1, ph_a1) : wait_group(2, kIssuer, bar_a, ph_a0)))
                 return;
             a_build(smem, tmem, par);
             fence_proxy_async_smem();
@@ -1010,20 +1037,12 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             fast = guard(state_max() + 64.0f * mk_cur * mv_cur);
             if (tid == kIssuer) {
                 sMisc[2] = fast ? 1u : 0u;
-                if (!fast) {
+                if (!fast)
                     mbar_arrive(bar_go);
-                } else {
-                    const uint32_t nsetb = sb + (uint32_t)par * SET_BYTES;
-#pragma unroll 1
-                    for (int kk = 0; kk < D / 16; ++kk) {
-                        const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
-                        mma_f16_ss(tmem + TM_A, sdesc_sw128(nsetb + S_QH + koff, 16, 1024),
-                                   sdesc_sw128(nsetb + S_KH + koff, 16, 1024), IDF_N64, kk > 0);
-                    }
-                }
             }
-            qk_issued = fast;
             stop_exact = !fast;
+            if (!fast && !(par ? wait_group(2, kIssuer, bar_a1, ph_a1) : wait_group(2, kIssuer, bar_a, ph_a0)))
+                return;
         }
         if (pend) {
             if (!wait_group(2, kIssuer, bar_o, ph_o))
@@ -1106,6 +1125,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             report(p.d_err, HS_DEVERR_TIMEOUT);
             if (n_tma > 0)
                 mbar_wait_bounded(bar_tma, (n_tma - 1) & 1, kTimeoutNs);
+            tc_commit(bar_ld);   // the D_A products this thread issued
+            mbar_wait_bounded(bar_ld, 0, kTimeoutNs);
         }
         if (tid == kIssuer) {
             tc_commit(bar_s);
