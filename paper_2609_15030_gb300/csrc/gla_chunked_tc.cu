@@ -463,8 +463,10 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
 
 
 // ---- output epilogue of a processed segment (state warps): D_O buffer `par` -> o (lane e,
-// 32 rows)
-__device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t tstride, int L, int par)
+// 32 rows per warp).  With `spare_issuer`, the warp of the MMA-issuing thread (warp 8) is
+// left out while it issues, and warp 12 (the same TMEM lane quarter) writes both halves.
+__device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t tstride, int L, int par,
+                                             bool spare_issuer)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool worker = warp >= 8;
@@ -472,22 +474,27 @@ __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t t
     const int colhalf = (warp >> 2) & 1;
     const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
 
-    if (!worker)
+    if (!worker || (spare_issuer && warp == 8))
         return;
-    float r[32];
-    const int ib = colhalf * 32;
-    tmem_ld32(tmem + lrow + (par ? TM_O1 : TM_O0) + ib, r);
-    tmem_wait_ld();
-    float *op = ob + (int64_t)ib * tstride + e_own;
-    if (L == CH) {
+    const int h0 = (spare_issuer && warp == 12) ? 0 : colhalf;
+    const int h1 = (spare_issuer && warp == 12) ? 2 : colhalf + 1;
+#pragma unroll 1
+    for (int hh = h0; hh < h1; ++hh) {
+        float r[32];
+        const int ib = hh * 32;
+        tmem_ld32(tmem + lrow + (par ? TM_O1 : TM_O0) + ib, r);
+        tmem_wait_ld();
+        float *op = ob + (int64_t)ib * tstride + e_own;
+        if (L == CH) {
 #pragma unroll
-        for (int x = 0; x < 32; ++x)
-            __stcs(op + (int64_t)x * tstride, r[x]);
-    } else {
-#pragma unroll
-        for (int x = 0; x < 32; ++x)
-            if (ib + x < L)
+            for (int x = 0; x < 32; ++x)
                 __stcs(op + (int64_t)x * tstride, r[x]);
+        } else {
+#pragma unroll
+            for (int x = 0; x < 32; ++x)
+                if (ib + x < L)
+                    __stcs(op + (int64_t)x * tstride, r[x]);
+        }
     }
 }
 
@@ -891,7 +898,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (!wait_all(kIssuer, bar_s, ph_s))
             return false;
         state_pass(smem, tmem, -1, ckpt_slot(seg_end), false);   // checkpoint and |S| of the final state
-        out_epilogue(tmem, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride, L, par);
+        out_epilogue(tmem, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride, L, par, false);
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -930,6 +937,11 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 return;
             const bool next_long = is_long(rpos + L);
             if (tid == kLoader) {
+                mbar_arrive(bar_built);
+                // the staged rows are consumed: stage the next segment (long or short) now;
+                // an exact decision on this one reloads it
+                if (rpos + L < end)
+                    issue_tma(rtok + L);
                 // D_A = Q~ K~^T of this segment, into its own buffer (the state warps wait on
                 // bar_a / bar_a1 by parity before they read it)
                 tc_fence_after();
@@ -941,11 +953,6 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                                sdesc_sw128(setb + S_KH + koff, 16, 1024), IDF_N64, kk > 0);
                 }
                 tc_commit(par ? bar_a1 : bar_a);
-                mbar_arrive(bar_built);
-                // the staged rows are consumed: stage the next segment (long or short) now;
-                // an exact decision on this one reloads it
-                if (rpos + L < end)
-                    issue_tma(rtok + L);
             }
             if (!wait_group(1, kLoader, bar_go, ph_go))
                 return;
@@ -1001,7 +1008,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 }
             }
             if (pend)
-                out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par);
+                out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par, true);
             // D_A of this segment (issued by the builders' loader)
             if (!(par ? wait_group(2, kIssuer, bar_a1, ph_a1) : wait_group(2, kIssuer, bar_a, ph_a0)))
                 return;
@@ -1048,7 +1055,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             if (!wait_group(2, kIssuer, bar_o, ph_o))
                 return;
             state_pass(smem, tmem, pend_g, ckpt_slot(pend_end), false);
-            out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par);
+            out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par, false);
             tc_fence_before();
             if (!sync_group(2))
                 return;
