@@ -165,6 +165,32 @@ def test_fp16_range_guards_take_the_exact_path(case):
         assert np.array_equal(ck_r[0].view(np.uint32), cks[0][m + 1:].view(np.uint32))
 
 
+@pytest.mark.parametrize("pattern", ["first", "middle_pair", "last", "all"])
+def test_exact_segments_at_run_boundaries(pattern):
+    """Segments sent to the exact path (growing gates) where a run of fast segments
+    would start, two in a row between two runs, at the last long segment before a
+    trailing short one, and everywhere; the call starts off the grid with a leading
+    short segment.  All match the oracle, and resuming on the grid from the call's own
+    checkpoint reproduces it bit for bit."""
+    dev = device()
+    pos0, N, C, nH, d = 60, 329, 64, 4, 128      # segments: 4 | 5 x 64 | 5 tokens
+    inp = gen_linear(21, 0, 1, N, nH, d, d)
+    S0 = gen_state(21, 0, 1, nH, d, d)
+    for k in {"first": [0], "middle_pair": [2, 3], "last": [4], "all": range(5)}[pattern]:
+        inp.a[:, 4 + 64 * k:4 + 64 * (k + 1)] = 0.02
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [pos0], [N], S0=S0, C_=C)
+    o, S, cks = run_prefill(inp, [pos0], [N], S0, C, dev, hs.HS_LINATTN_CHUNKED_TC)
+    _check(o, S, cks, ro, rS, rck, [pos0], [N], pattern)
+    c = 192
+    t, m = c - pos0, c // C - pos0 // C - 1
+    sub = type(inp)(*(x[:, t:N].copy() for x in (inp.q, inp.k, inp.v, inp.a)))
+    o_r, S_r, ck_r = run_prefill(sub, [c], [N - t], cks[0][m][None], C, dev,
+                                 hs.HS_LINATTN_CHUNKED_TC)
+    assert np.array_equal(o_r[0, :N - t].view(np.uint32), o[0, t:N].view(np.uint32))
+    assert np.array_equal(S_r.view(np.uint32), S.view(np.uint32))
+    assert np.array_equal(ck_r[0].view(np.uint32), cks[0][m + 1:].view(np.uint32))
+
+
 @pytest.mark.parametrize("kernel", KERNELS)
 def test_decode_steps_continue_the_prefill(kernel):
     """Hybrid workload shape: tail prefill then single-token decode steps off the grid."""
