@@ -21,7 +21,7 @@ timed on the host cores as a CPU baseline.
 ``--impl reference`` times the oracle itself (CPU) on a bounded sample of
 the same workload.
 
-``--case decode|prefill|kv`` runs one small piece of the workload a few
+``--case decode|prefill|kv|ckpt`` runs one small piece of the workload a few
 times and prints its CUDA-event times (no JSON): the cases the committed ncu
 captures under profiles/ were taken on.  ``--case long`` prints resumed vs
 recomputed TTFT for the long-context stack (L = 16k/32k/64k, batch 4).
@@ -612,6 +612,45 @@ def kv_host(dev, save=False, n_requests=8, pool=2):
     return out
 
 
+def state_copy(dev, reps=20, pool=8):
+    """The standalone checkpoint writer (hs_checkpoint_states; hs_restore_state is the same
+    copy the other way) on the long-context stack's live states: 4 requests x 18 linear
+    layers, 32 heads x 128 x 128 float32 each (2 MiB per layer, 144 MiB per snapshot), into
+    checkpoint slots rotating over `pool` snapshots (1.2 GB) from two rotating live sets, so
+    neither side stays in L2."""
+    import torch
+    import paper_2609_15030_gb300 as hs
+    from hs_inputs import LONG24
+    S = LONG24
+    n = S.batch * S.n_lin
+    floats = S.n_heads * S.d * S.d
+    live = torch.randn((2, n, floats), device=dev)
+    slots = torch.empty((pool, n, floats), device=dev)
+    live_ptrs = [hs.ptr_array([live[j, i] for i in range(n)], dev) for j in range(2)]
+    slot_ptrs = [hs.ptr_array([slots[j, i] for i in range(n)], dev) for j in range(pool)]
+    stream = torch.cuda.current_stream(dev)
+    for i in range(3):
+        hs.hs_checkpoint_states(live_ptrs[i % 2], slot_ptrs[i % pool], n, floats, None, stream.cuda_stream)
+    torch.cuda.synchronize(dev)
+    evs = []
+    for i in range(reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        hs.hs_checkpoint_states(live_ptrs[i % 2], slot_ptrs[(i + 3) % pool], n, floats, None,
+                                stream.cuda_stream)
+        e1.record(stream)
+        evs.append((e0, e1))
+    torch.cuda.synchronize(dev)
+    ok = torch.equal(slots[(reps - 1 + 3) % pool], live[(reps - 1) % 2])
+    t = statistics.median(e0.elapsed_time(e1) for e0, e1 in evs) * 1e-3
+    nb = 2 * n * floats * 4
+    del live, slots
+    return {"bytes_per_call": nb, "median_us": round(t * 1e6, 2), "gbs": round(nb / t / 1e9, 1),
+            "states": f"{n} x {floats * 4 // 2 ** 20} MiB (4 requests x 18 layers x 32 heads)",
+            "copy_checked": bool(ok)}
+
+
 def kv_rank_slices(dev, n_requests=16):
     """One tensor-parallel rank's restore of FP8 KV pages (Table 1: TP=4, FP8 KV): 48
     layers x 256 pages of 16 tokens x 8 KV heads x 128 (one byte each, 32 KiB pages);
@@ -831,7 +870,8 @@ def run_case(name: str, iters: int = 5):
     """decode: 64 single-token calls over 9 problems x 16 heads (d = 128);
     prefill: one 256-token tail over 9 problems x 16 heads from pos0 = 4096 with
     checkpoints every 256; kv: 12 layers x 256 pages x 64 KiB scattered into a
-    2,048-block cache.  Each repeated `iters` times on the current stream."""
+    2,048-block cache; ckpt: the standalone checkpoint writer on the long-context stack's
+    live states (72 x 2 MiB).  Each repeated `iters` times on the current stream."""
     import torch
     import paper_2609_15030_gb300 as hs
     from hs_inputs import torch_gen_linear, gen_block_table
@@ -880,6 +920,10 @@ def run_case(name: str, iters: int = 5):
             t = ev[0].elapsed_time(ev[1]) * 1e-3
             print(f"kv iter {it}: {t * 1e6:.1f} us, {kv_bytes(nL, n_pages, P) / t / 1e9:.0f} GB/s",
                   flush=True)
+    elif name == "ckpt":
+        for it in range(iters):
+            r = state_copy(dev, reps=4)
+            print(f"ckpt iter {it}: {r['median_us']:.1f} us, {r['gbs']:.0f} GB/s", flush=True)
     elif name == "long":
         return run_long(dev)
     else:
@@ -1008,7 +1052,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true",
                     help="skip TTFT arms, KV stress, e2e and CPU baseline")
-    ap.add_argument("--case", choices=["decode", "prefill", "kv", "long"],
+    ap.add_argument("--case", choices=["decode", "prefill", "kv", "ckpt", "long"],
                     help="run one small standalone case for a profiler capture")
     args = ap.parse_args()
     if args.case:
@@ -1120,6 +1164,10 @@ def main():
         sl = kv_rank_slices(dev)
         sl["frac"] = round(sl["gbs"] / peak, 4)
         out["kv_restore_rank_slice_fp8"] = sl
+        sc = state_copy(dev)
+        sc["frac"] = round(sc["gbs"] / peak, 4)
+        sc["traffic"] = _traffic().get("slot_copy_kernel@long24")
+        out["checkpoint_writer"] = sc
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
         print(json.dumps(out))

@@ -4,7 +4,8 @@
 //
 // Each slot is split into 64 KiB pieces so that a handful of large states
 // still spreads over every SM.  16-byte aligned slot pairs take 16-byte
-// vector loads/stores; any other pair falls back to 4-byte accesses.
+// vector loads/stores, eight in flight per thread before the first store;
+// any other pair falls back to 4-byte accesses.
 #include "hs_internal.cuh"
 
 namespace hs {
@@ -12,7 +13,7 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int64_t kPieceFloats = 16384;  // 64 KiB
-constexpr int kUnroll = 4;
+constexpr int kUnroll = 8;
 
 __global__ void __launch_bounds__(kThreads)
 slot_copy_kernel(const float *const *src, float *const *dst, int32_t n, int64_t floats_each,
