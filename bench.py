@@ -96,6 +96,19 @@ def _traffic():
     return out
 
 
+def _tensor_pipe():
+    """Tensor-pipe utilisation (of active, of elapsed cycles) from the committed ncu captures
+    listed in profiles/tensor_pipe.txt."""
+    p = os.path.join(ROOT, "profiles", "tensor_pipe.txt")
+    out = {}
+    if os.path.exists(p):
+        for line in open(p):
+            f = line.split()
+            if len(f) >= 3 and not line.startswith("#"):
+                out[f[0]] = {"active": float(f[1]), "elapsed": float(f[2]), "source": "ncu " + f[3]}
+    return out
+
+
 # ---------------------------------------------------------------------------
 # clocks sampler
 # ---------------------------------------------------------------------------
@@ -1120,15 +1133,20 @@ def main():
     groups = wl.step_phase_times() if whole else timer.summary()
     traffic = _traffic()
 
+    tensor = _tensor_pipe()
+
     def roofline(phase):
         nb, ms, n = groups[phase]
         ach = nb / (ms * 1e-3) / 1e9
         kern = KERNEL_OF[phase]
-        return {"bound": "hbm", "kernel": kern, "phase": phase, "achieved": round(ach, 1),
-                "peak": peak, "unit": "GB/s", "frac": round(ach / peak, 4), "peak_kind": peak_kind,
-                "traffic": traffic.get(kern), "bytes_per_launch": int(nb / n),
-                "avg_launch_us": round(ms * 1e3 / n, 3), "launches": n,
-                "share_of_step": round(ms * 1e-3 / t_phases, 3)}
+        r = {"bound": "hbm", "kernel": kern, "phase": phase, "achieved": round(ach, 1),
+             "peak": peak, "unit": "GB/s", "frac": round(ach / peak, 4), "peak_kind": peak_kind,
+             "traffic": traffic.get(kern), "bytes_per_launch": int(nb / n),
+             "avg_launch_us": round(ms * 1e3 / n, 3), "launches": n,
+             "share_of_step": round(ms * 1e-3 / t_phases, 3)}
+        if kern in tensor:
+            r["tensor_pipe_frac"] = tensor[kern]
+        return r
 
     dominant = max(groups, key=lambda k: groups[k][1])
     out = {
