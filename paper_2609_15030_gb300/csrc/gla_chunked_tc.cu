@@ -20,11 +20,13 @@
 // accumulators:  D_O = S^T Q~^T (A operand: an fp16 copy of S^T in TMEM),
 // D_A = Q~ K~^T, then [D_O | S^T] += V^T [A ; K~^T]^T as one N=192 product
 // (V^T in TMEM).  fp16 keeps the 10-bit mantissa of tf32 but halves the
-// instructions (K = 16 per MMA).  Two operand sets alternate, so while the
-// tensor core runs chunk c the eight operand warps stage chunk c+1 (cumulative
-// decay scan, Q~, K~, K~^T, V^T); the state pass between chunks applies the
-// pending decay 2^{Lam_last}, writes a due checkpoint and refreshes the fp16
-// copy of S^T.  One more warp issues every MMA and TMA copy.
+// instructions (K = 16 per MMA).  The CTA's 16 warps form two groups in a
+// pipeline over two alternating operand sets: while the eight state warps
+// finish chunk c (the state pass, which applies the pending decay 2^{Lam_last},
+// writes a due checkpoint and refreshes the fp16 copy of S^T; the causal mask;
+// the output epilogue) the eight builder warps stage chunk c+1 and build its
+// operands (cumulative decay scan, Q~, K~, K~^T, V^T).  The first builder thread
+// issues the TMA copies and D_A, the first state thread the other MMAs.
 //
 // A chunk is fast only if every fp16 operand provably stays below 2^15 in
 // magnitude: |q|, |v|, |K~|, the bound 128 max|q| max|k| on |A|, and a bound
@@ -38,9 +40,10 @@
 // most 8 tokens run the per-token recurrence with the recurrent kernel's exact
 // operation order.
 //
-// Every wait on an mbarrier is bounded (1 s); on timeout the CTA reports
-// HS_DEVERR_TIMEOUT, waits (bounded) for its own copies and MMAs in flight,
-// frees its TMEM and returns.
+// Every wait on an mbarrier is bounded (1 s) and is followed by a barrier that
+// reduces the abort flag, so every thread of a group takes the same branch; on
+// timeout the CTA reports HS_DEVERR_TIMEOUT, waits (bounded) for its own copies
+// and MMAs in flight, frees its TMEM and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
