@@ -12,8 +12,9 @@ namespace hs {
 // Programmatic dependent launch: every kernel of the library is launched with
 // programmatic stream serialization, so the next launch on the stream can be
 // scheduled while this one runs.  Each kernel waits for its predecessors to
-// complete (and their memory to be visible) before it touches global memory,
-// then releases its own dependents.
+// complete (and their memory to be visible) before it touches global memory
+// (L2 prefetches aside), then releases its own dependents; the tensor-core
+// prefill only waits (see pdl_wait).
 __device__ __forceinline__ void pdl_wait_and_release()
 {
     asm volatile("griddepcontrol.wait;" ::: "memory");
