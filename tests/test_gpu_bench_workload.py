@@ -23,7 +23,7 @@ def _bits(t):
     return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
 
 
-@pytest.mark.parametrize("r", [0, 8])            # L = 512 and L = 4608
+@pytest.mark.parametrize("r", range(9))          # L = 512, 1024, ..., 4608
 def test_hybrid_workload_request_matches_oracle(r):
     dev = device()
     import bench

@@ -12,8 +12,8 @@ import torch
 
 import oracle
 import paper_2609_15030_gb300 as hs
-from hs_inputs import (LONG24, SWEEP, TINY, bf16_bits_to_f32, f32_to_bf16_bits, gen_linear,
-                       gen_state)
+from hs_inputs import (LONG24, SWEEP, SWEEP_LENGTHS, TINY, bf16_bits_to_f32, f32_to_bf16_bits,
+                       gen_linear, gen_state)
 from tests.gpu_helpers import TOL, device, maxnorm_err, run_prefill, to_dev
 
 pytestmark = pytest.mark.gpu
@@ -69,7 +69,7 @@ def test_tiny_hybrid_config(kernel):
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
-@pytest.mark.parametrize("L", [512, 1536, 4608])
+@pytest.mark.parametrize("L", SWEEP_LENGTHS)
 def test_sweep_config_complete_and_partial_hit(kernel, L):
     """Single-layer sweep: 16 heads, d=128, C=512; complete hit and hit = L-37."""
     dev = device()
