@@ -12,8 +12,8 @@ import torch
 
 import oracle
 import paper_2609_15030_gb300 as hs
-from hs_inputs import (LONG24, SWEEP, SWEEP_LENGTHS, TINY, bf16_bits_to_f32, f32_to_bf16_bits,
-                       gen_linear, gen_state)
+from hs_inputs import (LONG24, LONG_LENGTHS, SWEEP, SWEEP_LENGTHS, TINY, bf16_bits_to_f32,
+                       f32_to_bf16_bits, gen_linear, gen_state)
 from tests.gpu_helpers import TOL, device, maxnorm_err, run_prefill, to_dev
 
 pytestmark = pytest.mark.gpu
@@ -280,13 +280,14 @@ def test_checkpoint_slot_errors_are_reported(kernel):
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
-def test_long_context_full_size_sampled_heads(kernel):
-    """Long-context stack shape at L = 16384: batch 4, 32 heads, d=128, C=512,
-    inputs drawn on the device; sampled (request, head) pairs against the oracle,
+@pytest.mark.parametrize("L", LONG_LENGTHS)
+def test_long_context_full_size_sampled_heads(kernel, L):
+    """Long-context stack shape at L = 16384, 32768 and 65536: batch 4, 32 heads, d=128,
+    C=512, inputs drawn on the device; sampled (request, head) pairs against the oracle,
     and the resumed tail (hit = L-37) bitwise against the full recomputation."""
     dev = device()
     from hs_inputs import torch_gen_linear
-    L, C, B, nH, d = 16384, LONG24.ckpt, LONG24.batch, LONG24.n_heads, LONG24.d
+    C, B, nH, d = LONG24.ckpt, LONG24.batch, LONG24.n_heads, LONG24.d
     q, k, v, a = torch_gen_linear(11, 0, B, L, nH, d, dev)
     state = torch.zeros((B, nH, d, d), device=dev)
     o = torch.zeros((B, L, nH, d), device=dev)
