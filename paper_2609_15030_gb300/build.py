@@ -7,6 +7,7 @@ HS_ERR_CUDA).
 """
 from __future__ import annotations
 
+import fcntl
 import os
 import subprocess
 import sys
@@ -47,7 +48,18 @@ def _stale(target, deps):
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
+    """Compile what is stale and link libhs.so.  Processes that build at the same time (one
+    per GPU under torchrun) take turns on a lock file, so none reads a half-written object."""
     os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            return _build_locked(force, verbose, extra_flags)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(force, verbose, extra_flags) -> str:
     nvcc = _nvcc()
     srcs = sources()
     hdrs = _deps()
