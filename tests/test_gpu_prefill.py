@@ -191,6 +191,30 @@ def test_exact_segments_at_run_boundaries(pattern):
     assert np.array_equal(ck_r[0].view(np.uint32), cks[0][m + 1:].view(np.uint32))
 
 
+@pytest.mark.parametrize("case", range(16))
+def test_random_configurations(case):
+    """Seeded random calls: batch 1-3, 1-3 heads, resume points anywhere in [0, 320), tails
+    of 0-399 tokens, checkpoint interval 0/64/128/192, from a random state, with growing
+    gates (the exact path) on up to two random token ranges; the tensor-core kernel and
+    AUTO against the oracle."""
+    dev = device()
+    rng = np.random.default_rng(1000 + case)
+    B, nH, d = int(rng.integers(1, 4)), int(rng.integers(1, 4)), 128
+    C = int(rng.choice([0, 64, 128, 192]))
+    pos0 = [int(x) for x in rng.integers(0, 320, B)]
+    n_tok = [int(x) for x in rng.integers(0, 400, B)]
+    T = max(max(n_tok), 1)
+    inp = gen_linear(2000 + case, 0, B, T, nH, d, d)
+    for _ in range(int(rng.integers(0, 3))):
+        b, t0 = int(rng.integers(B)), int(rng.integers(T))
+        inp.a[b, t0:t0 + int(rng.integers(1, 80))] = 0.02
+    S0 = gen_state(2000 + case, 0, B, nH, d, d)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, pos0, n_tok, S0=S0, C_=C, threads=8)
+    for kernel in (hs.HS_LINATTN_CHUNKED_TC, hs.HS_LINATTN_AUTO):
+        o, S, cks = run_prefill(inp, pos0, n_tok, S0, C, dev, kernel)
+        _check(o, S, cks, ro, rS, rck, pos0, n_tok, f"case {case} kernel {kernel}")
+
+
 @pytest.mark.parametrize("kernel", KERNELS)
 def test_decode_steps_continue_the_prefill(kernel):
     """Hybrid workload shape: tail prefill then single-token decode steps off the grid."""
