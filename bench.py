@@ -938,13 +938,14 @@ def run_case(name: str, iters: int = 5):
             r = state_copy(dev, reps=4)
             print(f"ckpt iter {it}: {r['median_us']:.1f} us, {r['gbs']:.0f} GB/s", flush=True)
     elif name == "long":
-        return run_long(dev)
+        run_long(dev)
+        return 0
     else:
         raise SystemExit(f"unknown case {name}")
     return 0
 
 
-def run_long(dev):
+def run_long(dev, reps=3, quiet=False):
     """Long-context hybrid stack: 24 layers (18 linear: 32 heads, d = 128, C = 512;
     6 full: 8 KV heads, head_dim 128, page 32), batch 4, L in {16k, 32k, 64k},
     complete hit (c = L - 512) and partial hit L - 37 (same c).  Resumed TTFT =
@@ -952,7 +953,8 @@ def run_long(dev):
     512-token tail prefill of every linear layer; recomputation = prefill of
     [0,L) from the zero state emitting every checkpoint + the KV write of L
     tokens.  One q/k/v/gate set per request is shared by the 18 linear layers
-    (18 distinct sets at L = 64k would need ~190 GB), so each layer is one call."""
+    (18 distinct sets at L = 64k would need ~190 GB), so each layer is one call.
+    Medians of `reps` timed runs after one warm-up; returns one row per case."""
     import torch
     import paper_2609_15030_gb300 as hs
     from hs_inputs import LONG24, LONG_LENGTHS, torch_gen_linear, torch_fill_bf16_normal
@@ -978,7 +980,9 @@ def run_long(dev):
     src_ptrs = hs.ptr_array([ck_src[l] for l in range(nL)], dev)
     dst_ptrs = hs.ptr_array([states[l] for l in range(nL)], dev)
     ev = lambda: torch.cuda.Event(enable_timing=True)
-    print(json.dumps({"case": "long", "workload": "long-24L (18 linear 32h d128 C512 + 6 full 8kv hd128 P32), batch 4"}))
+    rows = []
+    if not quiet:
+        print(json.dumps({"case": "long", "workload": "long-24L (18 linear 32h d128 C512 + 6 full 8kv hd128 P32), batch 4"}))
     for Lc in LONG_LENGTHS:
         # complete hit; cached prefix L-37 of an L-token prompt; an (L-37)-token prompt
         # fully cached (ragged tail inside the last chunk)
@@ -1011,16 +1015,23 @@ def run_long(dev):
             for nm, fn in (("resume", resume), ("recompute", recompute)):
                 fn()
                 torch.cuda.synchronize(dev)
-                e0, e1 = ev(), ev()
-                e0.record()
-                fn()
-                e1.record()
-                torch.cuda.synchronize(dev)
-                res[nm] = e0.elapsed_time(e1)
-            print(json.dumps({"L": L, "hit": hit, "c": c, "tail": tail, "ttft_resume_ms": round(res["resume"], 3),
-                              "ttft_recompute_ms": round(res["recompute"], 3),
-                              "ratio": round(res["recompute"] / res["resume"], 1)}), flush=True)
-    return 0
+                ts = []
+                for _ in range(reps):
+                    e0, e1 = ev(), ev()
+                    e0.record()
+                    fn()
+                    e1.record()
+                    torch.cuda.synchronize(dev)
+                    ts.append(e0.elapsed_time(e1))
+                res[nm] = statistics.median(ts)
+            row = {"L": L, "hit": hit, "c": c, "tail": tail, "ttft_resume_ms": round(res["resume"], 3),
+                   "ttft_recompute_ms": round(res["recompute"], 3),
+                   "ratio": round(res["recompute"] / res["resume"], 1)}
+            rows.append(row)
+            if not quiet:
+                print(json.dumps(row), flush=True)
+    del q, k, v, a, o, states, slots, cache, staging, ck_src
+    return rows
 
 
 # ---------------------------------------------------------------------------
@@ -1186,6 +1197,8 @@ def main():
         sc["frac"] = round(sc["gbs"] / peak, 4)
         sc["traffic"] = _traffic().get("slot_copy_kernel@long24")
         out["checkpoint_writer"] = sc
+        torch.cuda.empty_cache()
+        out["ttft_long_ms"] = run_long(dev, quiet=True)
         out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
         print(json.dumps(out))
