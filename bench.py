@@ -316,7 +316,9 @@ class Hybrid12:
         timing events are recorded between phases inside the graph, so the per-phase
         times are device times of the kernels themselves; each such event also ends
         the programmatic launch chain across its phase boundary (~5 us per boundary),
-        so the headline step time is taken on the graphs without them.  Returns False
+        so the headline step time is taken on the graphs without them.  Without events
+        only one graph per seed is captured (steps replay them in rotation); with events
+        every step has its own graph, whose events keep that step's times.  Returns False
         (nothing captured) where this PyTorch cannot record events inside a graph."""
         torch = self.torch
         if events:
@@ -326,7 +328,7 @@ class Hybrid12:
                 return False
         side = torch.cuda.Stream(self.dev)
         graphs = []
-        for i in range(n):
+        for i in range(n if events else min(n, self.seeds)):
             s = i % self.seeds
             g = torch.cuda.CUDAGraph()
             marks, launches = [], 0
@@ -1071,7 +1073,7 @@ def aggregate_value(tokens_per_rank_step: int, steps: int, world_size: int, t_ma
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true",
