@@ -66,6 +66,11 @@ constexpr int kLoader = 0;   // the first builder thread issues every TMA copy
 constexpr int kIssuer = NB;  // the first state thread issues every MMA
 constexpr int kShort = 8; // segments of at most this many tokens run token by token
 constexpr float kLog2e = 1.4426950408889634f;
+// exact path: log-gates below this are taken at this value.  2^(kGateFloor * log2 e) = 2^-144
+// is flushed to 0 by ex2.approx.ftz, so such a gate still zeroes the state, while the
+// cumulative log2-decay after it stays small enough (|Lam| of a few hundred, not ~1.4e4 for
+// a gate of -1e4) for the differences Lam_i - Lam_j of later tokens to keep their precision.
+constexpr float kGateFloor = -100.0f;
 constexpr float kF16Lim = 32768.0f;         // fast-path fp16 operands stay below 2^15
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr int kPrefetch = 2;                // segments requested into L2 ahead of the staged one
@@ -799,7 +804,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             if (worker) {
 #pragma unroll 8
                 for (int x = 0; x < 32; ++x) {
-                    run = fmaf(sG[(32 * th + x) * D + d], kLog2e, run);
+                    run = fmaf(fmaxf(sG[(32 * th + x) * D + d], kGateFloor), kLog2e, run);
                     sLam[(32 * th + x) * D + d] = run;
                 }
                 sTot[th * D + d] = run;

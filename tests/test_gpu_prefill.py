@@ -191,6 +191,30 @@ def test_exact_segments_at_run_boundaries(pattern):
     assert np.array_equal(ck_r[0].view(np.uint32), cks[0][m + 1:].view(np.uint32))
 
 
+@pytest.mark.parametrize("where", ["short_call", "full_segment"])
+def test_zero_gate_inside_an_exact_segment(where):
+    """A zero gate (a = -1e4) followed, in the same segment, by growing gates (the exact
+    path): the decay factors of the tokens after the zero gate are differences of
+    cumulative log-gates, which must stay accurate (the state is reset by the zero gate
+    and then grows).  Outputs and final state against the oracle."""
+    dev = device()
+    nH, d, C = 2, 128, 512
+    if where == "short_call":
+        pos0, n = 221, 18                  # one 18-token segment inside a chunk
+        z, g0, g1 = 7, 2, 18
+    else:
+        pos0, n = 192, 64                  # one whole chunk
+        z, g0, g1 = 10, 11, 64
+    inp = gen_linear(60250, 0, 1, n, nH, d, d)
+    inp.a[0, g0:g1] = 0.02
+    inp.a[0, z] = -1e4
+    S0 = gen_state(60250, 0, 1, nH, d, d) * 100.0
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [pos0], [n], S0=S0, C_=C)
+    for kernel in (hs.HS_LINATTN_CHUNKED_TC, hs.HS_LINATTN_AUTO):
+        o, S, cks = run_prefill(inp, [pos0], [n], S0, C, dev, kernel)
+        _check(o, S, cks, ro, rS, rck, [pos0], [n], f"{where} kernel {kernel}")
+
+
 @pytest.mark.parametrize("case", range(16))
 def test_random_configurations(case):
     """Seeded random calls: batch 1-3, 1-3 heads, resume points anywhere in [0, 320), tails
