@@ -29,8 +29,9 @@
 // issues the TMA copies and D_A, the first state thread the other MMAs.
 //
 // A chunk is fast only if every fp16 operand provably stays below 2^15 in
-// magnitude: |q|, |v|, |K~|, the bound 128 max|q| max|k| on |A|, and a bound
-// on |S| carried from the measured state.  Any other chunk (strong decay,
+// magnitude (|q|, |v|, |K~|, the bound 128 max|q| max|k| on |A|, and a bound
+// on |S| carried from the measured state) and its total decay is at most 2^-10
+// in every key dim (so Q~ never nears fp16's subnormals).  Any other chunk (strong decay,
 // huge values) runs the exact path: tf32 operands, the intra-chunk matrix
 // computed elementwise with 2^{Lam_i - Lam_j} <= 1, and the state updated as
 // diag(2^{Lam_last}) S + K^^T V with K^_j = k_j 2^{Lam_last - Lam_j}.  The
@@ -72,6 +73,8 @@ constexpr float kLog2e = 1.4426950408889634f;
 // a gate of -1e4) for the differences Lam_i - Lam_j of later tokens to keep their precision.
 constexpr float kGateFloor = -100.0f;
 constexpr float kF16Lim = 32768.0f;         // fast-path fp16 operands stay below 2^15
+constexpr float kLamRange = 10.0f;          // fast path: a segment's total log2-decay >= -10, so
+                                            // Q~ = q 2^Lam stays far from fp16's subnormals
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr int kPrefetch = 2;                // segments requested into L2 ahead of the staged one
 
@@ -109,6 +112,11 @@ constexpr uint32_t TM_SH = 256;         // S^T fp16 copy, two key dims per colum
 constexpr uint32_t TM_A0 = 320;         // D_A of even segments, 128 lanes x 64 cols (lanes 0..63 used)
 constexpr uint32_t TM_V = 384;          // V^T: fast, fp16 pairs 2 x 32 cols; exact, f32 64 cols
 constexpr uint32_t TM_A1 = 448;         // D_A of odd segments
+// exact path (no fast-path data live): S^T as two tf32 parts for S^T Q~^T, hi in the 128
+// columns of D_O1 and the fp16 copy, lo in the two D_A buffers (key dims 0..63, 64..127)
+constexpr uint32_t TM_SHI = 192;
+constexpr uint32_t TM_SLO0 = 320;
+constexpr uint32_t TM_SLO1 = 448;
 
 constexpr uint32_t IDF_N64 = idesc_f16(128, 64);
 constexpr uint32_t IDF_N192 = idesc_f16(128, 192);
@@ -289,6 +297,7 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
     bar_builders();
     // the running sums start from the earlier quarters' totals
     float run0 = 0.f, run1 = 0.f;
+    bool lam_ok;
     {
         float t0 = 0.f, t1 = 0.f;
 #pragma unroll
@@ -303,6 +312,7 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
         }
         if (qt == 0)
             *reinterpret_cast<float2 *>(sGam + gslot * D + 2 * dp) = make_float2(ex2(t0), ex2(t1));
+        lam_ok = t0 >= -kLamRange && t1 >= -kLamRange;
     }
     uint8_t *set = smem + par * SET_BYTES;
     const int rowK = par ? 0 : 64;
@@ -360,9 +370,11 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
     float mq = warp_max(bmax_of(bq));
     float mk = warp_max(bmax_of(bk));
     float mv = warp_max(bmax_of(bv));
-    // non-increasing Lam (|Q~| <= |q|, |A| <= 128 max|q| max|k|) and every fp16 operand
-    // below 2^15; NaN fails
-    bool ok = amax <= 0.f && hmax_of(hq) < kF16Lim && hmax_of(hk) < kF16Lim && mv < kF16Lim;
+    // non-increasing Lam (|Q~| <= |q|, |A| <= 128 max|q| max|k|), a total decay of at most
+    // 2^-10 (Q~ of the segment's last tokens keeps its precision) and every fp16 operand below
+    // 2^15; NaN fails
+    bool ok = amax <= 0.f && lam_ok && hmax_of(hq) < kF16Lim && hmax_of(hk) < kF16Lim &&
+              mv < kF16Lim;
     ok = __all_sync(0xffffffffu, ok);
     if (lane == 0) {
         sRed[warp * 8 + 0] = mq;
@@ -845,20 +857,45 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 }
                 tmem_st16(tmem + lrow + TM_V + 32 * th + 16 * hh, vtr);
             }
+            // the state as two tf32 parts for S^T Q~^T (an A operand from TMEM is read as
+            // tf32): hi = S with its low 13 mantissa bits cleared (exact in tf32), lo = S - hi
+            // (exact in fp32, at most 13 significant bits), so the product keeps the state to
+            // ~2^-20 instead of a 2^-10 truncation
+#pragma unroll 1
+            for (int c0 = 0; c0 < 64; c0 += 32) {
+                const int d0 = colhalf * 64 + c0;
+                float r[32], lo[32];
+                tmem_ld32(tmem + lrow + TM_S + d0, r);
+                tmem_wait_ld();
+#pragma unroll
+                for (int x = 0; x < 32; ++x) {
+                    const float hi = __uint_as_float(__float_as_uint(r[x]) & 0xFFFFE000u);
+                    lo[x] = r[x] - hi;
+                    r[x] = hi;
+                }
+                tmem_st32(tmem + lrow + TM_SHI + d0, r);
+                tmem_st32(tmem + lrow + (d0 < 64 ? TM_SLO0 + d0 : TM_SLO1 + (d0 - 64)), lo);
+            }
             tmem_wait_st();
         }
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
-        const uint32_t tm_o = par ? TM_O1 : TM_O0;
+        const uint32_t tm_o = TM_O0;   // par is 0 here: D_O1's columns hold the split state
         if (tid == kIssuer) {
-            // S^T Q~^T into D_O (A operand: the float32 state in TMEM)
+            // S^T Q~^T into D_O: the hi part, then the lo part
             tc_fence_after();
-#pragma unroll
+#pragma unroll 1
             for (int kk = 0; kk < D / 8; ++kk) {
                 const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
-                mma_tf32_ts(tmem + tm_o, tmem + TM_S + kk * 8, sdesc_sw128(sb + X_QT + koff, 16, 1024),
+                mma_tf32_ts(tmem + tm_o, tmem + TM_SHI + kk * 8, sdesc_sw128(sb + X_QT + koff, 16, 1024),
                             IDT_N64, kk > 0);
+            }
+#pragma unroll 1
+            for (int kk = 0; kk < D / 8; ++kk) {
+                const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
+                const uint32_t lo = kk < 8 ? TM_SLO0 + kk * 8 : TM_SLO1 + (kk - 8) * 8;
+                mma_tf32_ts(tmem + tm_o, tmem + lo, sdesc_sw128(sb + X_QT + koff, 16, 1024), IDT_N64, 1);
             }
         }
         // A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}, j <= i < L, elementwise
