@@ -215,6 +215,26 @@ def test_zero_gate_inside_an_exact_segment(where):
         _check(o, S, cks, ro, rS, rck, [pos0], [n], f"{where} kernel {kernel}")
 
 
+@pytest.mark.parametrize("n_strong", [6, 9, 12])
+def test_strong_decay_early_in_each_chunk(n_strong):
+    """The first n_strong tokens of every chunk carry a log-gate of -1.2, so each chunk's
+    total log2-decay is about -(10.4, 15.6, 20.8) - 4: around the fast path's limit of -10
+    (beyond it Q~ = q 2^Lam of the chunk's last tokens would sit in fp16's subnormal range)
+    and, for the larger two, past the fp16 range of K~.  Three chunks from a resumed
+    position with a checkpoint in the middle, both kernels against the oracle."""
+    dev = device()
+    nH, d, C = 2, 128, 128
+    pos0, n = 128, 192
+    inp = gen_linear(60300 + n_strong, 0, 1, n, nH, d, d)
+    for c0 in range(0, n, 64):
+        inp.a[0, c0:c0 + n_strong] = -1.2
+    S0 = gen_state(60300 + n_strong, 0, 1, nH, d, d)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [pos0], [n], S0=S0, C_=C)
+    for kernel in (hs.HS_LINATTN_CHUNKED_TC, hs.HS_LINATTN_AUTO):
+        o, S, cks = run_prefill(inp, [pos0], [n], S0, C, dev, kernel)
+        _check(o, S, cks, ro, rS, rck, [pos0], [n], f"n_strong {n_strong} kernel {kernel}")
+
+
 @pytest.mark.parametrize("case", range(16))
 def test_random_configurations(case):
     """Seeded random calls: batch 1-3, 1-3 heads, resume points anywhere in [0, 320), tails
