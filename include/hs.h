@@ -315,6 +315,14 @@ typedef struct hs_linattn_shape {
  *              position order; hs_linattn_num_checkpoints gives the count.  Each
  *              slot must be 16-byte aligned (else HS_DEVERR_MISALIGNED, not written).
  *   d_err      optional device int32 (see conventions)
+ * Accuracy: the recurrent and single-token kernels compute in float32 token by
+ * token.  The tensor-core kernel runs a chunk on fp16 operands (11 significant
+ * bits, float32 accumulation and state) when its log-gates are <= 0, its total
+ * log2-decay stays >= -10 in every key dimension and every operand provably fits
+ * fp16; any other chunk runs on tf32 operands with the intra-chunk scores computed
+ * in float32.  Against a float64 reference both stay within a max-normalised error
+ * of 2e-3 per (problem, head) unless a head's largest output is one score q_i.k_j
+ * whose terms cancel strongly, times a v_j far larger than the head's other values.
  * All of q, k, v, log_g, o, state must be 16-byte aligned.  q/k/v/log_g are only
  * read; o, state and the slots must not overlap the inputs or each other.
  * Token rows are 32-bit: b*max_tokens + n_tokens[b] must stay below 2^31.
