@@ -841,10 +841,16 @@ def cpu_baseline():
     t0 = time.perf_counter()
     toks = sum(s.run(cores) for s in samples)
     t = time.perf_counter() - t0
+    # the same oracle on one thread, for the first request only
+    t1 = time.perf_counter()
+    toks1 = samples[0].run(1)
+    t1 = time.perf_counter() - t1
     return {"value": round(toks / t, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
             "sample": f"one step (the 9 requests of seed 0): align + page scatter + state copy + "
                       "256-token tail and 64 decode tokens of all 9 linear layers x 16 heads, "
-                      f"float64 token by token; {t:.1f} s wall on {cores} threads"}
+                      f"float64 token by token; {t:.1f} s wall on {cores} threads",
+            "one_thread": {"value": round(toks1 / t1, 2), "unit": "tokens/s", "cores": 1,
+                           "sample": f"request 0 of the same step (L = 512) on one thread, {t1:.1f} s wall"}}
 
 
 def run_reference(args):
