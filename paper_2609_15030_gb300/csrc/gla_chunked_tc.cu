@@ -30,10 +30,12 @@
 //
 // A chunk is fast only if every fp16 operand provably stays below 2^15 in
 // magnitude (|q|, |v|, |K~|, the bound 128 max|q| max|k| on |A|, and a bound
-// on |S| carried from the measured state) and its total decay is at most 2^-10
-// in every key dim (so Q~ never nears fp16's subnormals).  Any other chunk (strong decay,
-// huge values) runs the exact path: tf32 operands, the intra-chunk matrix
-// computed elementwise with 2^{Lam_i - Lam_j} <= 1, and the state updated as
+// on |S| carried from the measured state) and its total decay factor
+// 2^{Lam_last} stays >= 2^-10 in every key dim (so Q~ never nears fp16's
+// subnormals).  Any other chunk (strong decay, huge values) runs the exact
+// path: tf32 operands (the state split into two exact tf32 parts), the
+// intra-chunk matrix computed elementwise in float32 with 2^{Lam_i - Lam_j} <= 1,
+// and the state updated as
 // diag(2^{Lam_last}) S + K^^T V with K^_j = k_j 2^{Lam_last - Lam_j}.  The
 // choice depends only on the chunk's inputs and on the state it starts from,
 // as does every operation order, so a resumed run reproduces a full
