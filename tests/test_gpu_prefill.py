@@ -235,6 +235,28 @@ def test_strong_decay_early_in_each_chunk(n_strong):
         _check(o, S, cks, ro, rS, rck, [pos0], [n], f"n_strong {n_strong} kernel {kernel}")
 
 
+@pytest.mark.parametrize("kernel", [hs.HS_LINATTN_AUTO, hs.HS_LINATTN_CHUNKED_TC,
+                                    hs.HS_LINATTN_RECURRENT, hs.HS_LINATTN_SINGLE_TOKEN])
+def test_largest_batch(kernel):
+    """HS_MAX_BATCH problems in one call (the largest launch parameter block): one head
+    each, random resume points and tails (one token each for the single-token kernel),
+    checkpoints every 64, from random states; every problem against the oracle."""
+    dev = device()
+    rng = np.random.default_rng(384)
+    B, nH, d, C = hs.HS_MAX_BATCH, 1, 128, 64
+    pos0 = [int(x) for x in rng.integers(0, 300, B)]
+    if kernel == hs.HS_LINATTN_SINGLE_TOKEN:
+        n_tok = [int(x) for x in rng.integers(0, 2, B)]
+    else:
+        n_tok = [int(x) for x in rng.integers(0, 100, B)]
+    T = max(max(n_tok), 1)
+    inp = gen_linear(384, 0, B, T, nH, d, d)
+    S0 = gen_state(384, 0, B, nH, d, d)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, pos0, n_tok, S0=S0, C_=C, threads=16)
+    o, S, cks = run_prefill(inp, pos0, n_tok, S0, C, dev, kernel)
+    _check(o, S, cks, ro, rS, rck, pos0, n_tok, f"batch {B} kernel {kernel}")
+
+
 @pytest.mark.parametrize("case", range(16))
 def test_random_configurations(case):
     """Seeded random calls: batch 1-3, 1-3 heads, resume points anywhere in [0, 320), tails
