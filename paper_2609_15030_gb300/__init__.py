@@ -43,7 +43,8 @@ HS_LINATTN_SINGLE_TOKEN = 3
 EXPORTED = ("hs_status_string", "hs_version", "hs_align_prefix", "hs_restore_kv_pages",
             "hs_save_kv_pages", "hs_restore_kv_page_slices", "hs_save_kv_page_slices",
             "hs_restore_state", "hs_checkpoint_states", "hs_linattn_prefill_from_state",
-            "hs_linattn_num_checkpoints", "hs_linattn_prefill_packed", "hs_restore_request")
+            "hs_linattn_num_checkpoints", "hs_linattn_prefill_packed", "hs_restore_request",
+            "hs_test_prefill_stalled")
 
 
 class HsError(RuntimeError):
@@ -89,6 +90,7 @@ def load() -> C.CDLL:
             L.hs_linattn_num_checkpoints.argtypes = [i32, vp, vp, i32, vp]
             L.hs_linattn_prefill_packed.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp, vp,
                                                     vp, vp, vp, vp, vp, i32, vp, vp, vp]
+            L.hs_test_prefill_stalled.argtypes = L.hs_linattn_prefill_from_state.argtypes
             for name in EXPORTED[2:]:
                 getattr(L, name).restype = C.c_int
             _lib = L
@@ -210,19 +212,31 @@ def make_shape(batch, n_heads, d_k, d_v, max_tokens, kernel=HS_LINATTN_AUTO):
                             int(kernel), 0)
 
 
+def _prefill_call(name, shape, q, k, v, log_g, o, state, pos0, n_tokens, ckpt_interval,
+                  ckpt_slots, d_err, stream):
+    B = int(shape.batch)
+    p0 = (C.c_int64 * max(B, 1))(*[int(x) for x in pos0])
+    nt = (C.c_int32 * max(B, 1))(*[int(x) for x in n_tokens])
+    rc = getattr(load(), name)(C.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(log_g), _ptr(o),
+                               _ptr(state), C.addressof(p0), C.addressof(nt), int(ckpt_interval),
+                               _ptr(ckpt_slots), _ptr(d_err), _stream(stream))
+    _check(rc, name)
+
+
 def hs_linattn_prefill_from_state(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0,
                                   n_tokens, ckpt_interval: int, ckpt_slots=None, d_err=None,
                                   stream=None):
     """pos0 / n_tokens: host sequences (ints) of length shape.batch."""
-    B = int(shape.batch)
-    p0 = (C.c_int64 * max(B, 1))(*[int(x) for x in pos0])
-    nt = (C.c_int32 * max(B, 1))(*[int(x) for x in n_tokens])
-    rc = load().hs_linattn_prefill_from_state(C.byref(shape), _ptr(q), _ptr(k), _ptr(v),
-                                              _ptr(log_g), _ptr(o), _ptr(state),
-                                              C.addressof(p0), C.addressof(nt),
-                                              int(ckpt_interval), _ptr(ckpt_slots), _ptr(d_err),
-                                              _stream(stream))
-    _check(rc, "hs_linattn_prefill_from_state")
+    _prefill_call("hs_linattn_prefill_from_state", shape, q, k, v, log_g, o, state, pos0,
+                  n_tokens, ckpt_interval, ckpt_slots, d_err, stream)
+
+
+def hs_test_prefill_stalled(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0, n_tokens,
+                            ckpt_interval: int, ckpt_slots=None, d_err=None, stream=None):
+    """Failure-detection hook (include/hs_test.h): the tensor-core prefill with one wait that
+    nothing completes; each CTA's bounded wait runs out and it reports HS_DEVERR_TIMEOUT."""
+    _prefill_call("hs_test_prefill_stalled", shape, q, k, v, log_g, o, state, pos0, n_tokens,
+                  ckpt_interval, ckpt_slots, d_err, stream)
 
 
 def hs_linattn_prefill_packed(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0, n_tokens,

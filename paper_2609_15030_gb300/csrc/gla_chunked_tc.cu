@@ -1114,8 +1114,17 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
     };
 
+    // failure-detection hook (tests only): every thread joins one CTA-wide wait on an
+    // mbarrier that nothing completes before the first decision (bar_go, phase 0); the
+    // loader's bounded wait runs out and raises the abort flag, and the CTA leaves through
+    // the abort path below
+    if (p.stall_for_test) {
+        uint32_t ph_stall = 0;
+        wait_all(kLoader, bar_go, ph_stall);
+    }
+
     int64_t pos = pos0, tok = 0;
-    while (pos < end) {
+    while (!aborted && pos < end) {
         const int L = seg_len(pos);
         if (L <= kShort) {
             // a leading or trailing short segment (its inputs are staged or in flight)

@@ -4,6 +4,7 @@
 #include <cstring>
 
 #include "hs_internal.cuh"
+#include "hs_test.h"
 
 namespace {
 
@@ -267,7 +268,7 @@ static hs_status prefill(const hs_linattn_shape *shp, const uint16_t *q, const u
                          const uint16_t *v, const float *log_g, float *o, float *state,
                          const int64_t *pos0, const int32_t *n_tokens, const int64_t *cu_rows,
                          int32_t ckpt_interval, float *const *ckpt_slots, int32_t *d_err,
-                         cudaStream_t stream)
+                         cudaStream_t stream, bool stall_for_test = false)
 {
     if (shp == nullptr)
         return HS_ERR_INVALID_ARG;
@@ -279,6 +280,8 @@ static hs_status prefill(const hs_linattn_shape *shp, const uint16_t *q, const u
         return HS_ERR_INVALID_ARG;
     if (s.d_k != s.d_v || (s.d_k != 64 && s.d_k != 128))
         return HS_ERR_UNSUPPORTED;
+    if (stall_for_test && s.kernel != HS_LINATTN_CHUNKED_TC)
+        return HS_ERR_UNSUPPORTED;   // the hook exists in the tensor-core kernel only
     if (s.batch > HS_MAX_BATCH)
         return HS_ERR_UNSUPPORTED;
     if (ckpt_interval < 0)
@@ -325,6 +328,7 @@ static hs_status prefill(const hs_linattn_shape *shp, const uint16_t *q, const u
     p.batch = s.batch;
     p.n_heads = s.n_heads;
     p.ckpt_interval = (p.ckpt_slots != nullptr) ? ckpt_interval : 0;
+    p.stall_for_test = stall_for_test ? 1 : 0;
     int64_t base = 0;
     for (int32_t b = 0; b < s.batch; ++b) {
         const int64_t r0 = cu_rows ? cu_rows[b] : (int64_t)b * s.max_tokens;
@@ -370,6 +374,16 @@ hs_status hs_linattn_prefill_from_state(const hs_linattn_shape *shp, const uint1
 {
     return prefill(shp, q, k, v, log_g, o, state, pos0, n_tokens, nullptr, ckpt_interval,
                    ckpt_slots, d_err, stream);
+}
+
+hs_status hs_test_prefill_stalled(const hs_linattn_shape *shp, const uint16_t *q,
+                                  const uint16_t *k, const uint16_t *v, const float *log_g,
+                                  float *o, float *state, const int64_t *pos0,
+                                  const int32_t *n_tokens, int32_t ckpt_interval,
+                                  float *const *ckpt_slots, int32_t *d_err, cudaStream_t stream)
+{
+    return prefill(shp, q, k, v, log_g, o, state, pos0, n_tokens, nullptr, ckpt_interval,
+                   ckpt_slots, d_err, stream, true);
 }
 
 hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t *q,

@@ -69,6 +69,7 @@ struct GlaParams {
     int32_t batch;
     int32_t n_heads;
     int32_t ckpt_interval;     // 0: none
+    int32_t stall_for_test;    // tensor-core kernel only: one wait that nothing completes (failure-detection tests)
     int64_t pos0[HS_MAX_BATCH];
     int32_t n_tokens[HS_MAX_BATCH];
     int32_t ck_base[HS_MAX_BATCH];  // index of the problem's first slot in ckpt_slots

@@ -1,10 +1,11 @@
 """Host-only checks of the C-ABI library (no GPU needed).
 
-* libhs.so loads and exports every function include/hs.h declares;
+* libhs.so loads and exports every function include/*.h declares;
 * hs_align_prefix (host integer code) matches the oracle bit-exactly;
 * every argument error is reported before any CUDA call.
 """
 import ctypes
+import glob
 import os
 import re
 
@@ -24,9 +25,11 @@ def built():
 
 
 def _declared():
-    txt = open(os.path.join(ROOT, "include", "hs.h")).read()
-    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
-    return sorted(set(re.findall(r"\b(hs_[a-z0-9_]+)\s*\(", txt)))
+    names = set()
+    for h in sorted(glob.glob(os.path.join(ROOT, "include", "*.h"))):
+        txt = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"\b(hs_[a-z0-9_]+)\s*\(", txt))
+    return sorted(names)
 
 
 def test_exports_every_declared_symbol():
@@ -220,6 +223,21 @@ def test_prefill_host_validation():
         assert e.value.status == code, kw
     call(shape_kw=dict(batch=0), pos0=[], n_tokens=[])    # empty batch: OK, nothing launched
     call(n_tokens=[0], q=None, k=None, v=None, log_g=None, o=None)   # empty tails: OK
+
+
+def test_stalled_prefill_hook_host_validation():
+    """The failure-detection hook exists in the tensor-core kernel only; other kernel
+    choices are refused on the host, and its argument checks are the prefill's."""
+    a = dict(q=FAKE, k=FAKE, v=FAKE, log_g=FAKE, o=FAKE, state=FAKE, pos0=[0], n_tokens=[8],
+             ckpt_interval=64, ckpt_slots=None, d_err=None, stream=0)
+    for kernel in (hs.HS_LINATTN_AUTO, hs.HS_LINATTN_RECURRENT, hs.HS_LINATTN_SINGLE_TOKEN):
+        with pytest.raises(hs.HsError) as e:
+            hs.hs_test_prefill_stalled(hs.make_shape(1, 2, 128, 128, 8, kernel), **a)
+        assert e.value.status == hs.HS_ERR_UNSUPPORTED
+    with pytest.raises(hs.HsError) as e:
+        hs.hs_test_prefill_stalled(hs.make_shape(1, 2, 128, 128, 8, hs.HS_LINATTN_CHUNKED_TC),
+                                   **dict(a, pos0=[-1]))
+    assert e.value.status == hs.HS_ERR_INVALID_ARG
 
 
 def test_packed_prefill_host_validation():
