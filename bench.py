@@ -83,6 +83,17 @@ KERNEL_OF = {"decode": "gla_decode_kernel<128>", "prefill": "gla_chunked_tc_kern
              "restore": "restore_request_kernel"}
 
 
+def _nvtx(name: str):
+    """An NVTX range around one section of the run (visible to ncu --nvtx and nsys);
+    a no-op context where torch has no NVTX support."""
+    import contextlib
+    try:
+        import torch
+        return torch.cuda.nvtx.range(name)
+    except Exception:
+        return contextlib.nullcontext()
+
+
 def _traffic():
     """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the
     committed ncu captures listed in profiles/dram_traffic.txt ("kernel bytes" lines)."""
@@ -1139,8 +1150,10 @@ def main():
     clocks.start()
     timer = LaunchTimer(torch, wl.stream)
     if whole:
-        t_local, launches = timed(False)
-        t_phases, _ = timed(True)
+        with _nvtx("hybrid12 timed steps"):
+            t_local, launches = timed(False)
+        with _nvtx("hybrid12 timed steps with phase events"):
+            t_phases, _ = timed(True)
     else:
         t_local, launches = timed(False, timer)
         t_phases = t_local
@@ -1186,28 +1199,36 @@ def main():
         "clocks": clk,
     }
     if rank == 0 and not args.no_extras:
-        wl_e2e = e2e_run(wl, args.steps, args.warmup)
+        with _nvtx("e2e through host buffers"):
+            wl_e2e = e2e_run(wl, args.steps, args.warmup)
         out["e2e"] = {k: wl_e2e[k] for k in ("value", "unit", "h2d_bytes_per_step", "d2h_bytes_per_step")}
         out["e2e"]["ms_per_step"] = wl_e2e["ms_per_step"]
-        out["ttft_us"] = ttft_arms(wl)
+        with _nvtx("ttft resume vs recompute"):
+            out["ttft_us"] = ttft_arms(wl)
         del wl
         torch.cuda.empty_cache()
-        kv = kv_stress(dev)
+        with _nvtx("kv stress"):
+            kv = kv_stress(dev)
         kv["frac"] = round(kv["gbs_aggregate"] / peak, 4)
         kv["traffic"] = _traffic().get("kv_scatter_kernel@kvstress")
         out["kv_restore"] = kv
-        out["kv_restore_from_host"] = kv_host(dev)
-        out["kv_save_to_host"] = kv_host(dev, save=True)
-        sl = kv_rank_slices(dev)
+        with _nvtx("kv host staging"):
+            out["kv_restore_from_host"] = kv_host(dev)
+            out["kv_save_to_host"] = kv_host(dev, save=True)
+        with _nvtx("kv rank slices"):
+            sl = kv_rank_slices(dev)
         sl["frac"] = round(sl["gbs"] / peak, 4)
         out["kv_restore_rank_slice_fp8"] = sl
-        sc = state_copy(dev)
+        with _nvtx("checkpoint writer"):
+            sc = state_copy(dev)
         sc["frac"] = round(sc["gbs"] / peak, 4)
         sc["traffic"] = _traffic().get("slot_copy_kernel@long24")
         out["checkpoint_writer"] = sc
         torch.cuda.empty_cache()
-        out["ttft_long_ms"] = run_long(dev, quiet=True)
-        out["cpu_baseline"] = cpu_baseline()
+        with _nvtx("long context"):
+            out["ttft_long_ms"] = run_long(dev, quiet=True)
+        with _nvtx("oracle baseline"):
+            out["cpu_baseline"] = cpu_baseline()
     if rank == 0:
         print(json.dumps(out))
     if ws > 1:
