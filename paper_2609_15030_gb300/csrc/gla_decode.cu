@@ -68,17 +68,18 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __
     const int64_t row = ((int64_t)p.row0[b]) * p.n_heads + h;   // the call's one token
     const uint4 *q8 = reinterpret_cast<const uint4 *>(p.q + row * D + 16 * rg);
     const uint4 *k8 = reinterpret_cast<const uint4 *>(p.k + row * D + 16 * rg);
-    const float4 *a4 = reinterpret_cast<const float4 *>(p.log_g + row * D + 16 * rg);
     const uint2 v2 = *reinterpret_cast<const uint2 *>(p.v + row * D + 4 * cg);
     uint32_t qw[8], kw[8];
-    float a[16];
     *reinterpret_cast<uint4 *>(&qw[0]) = q8[0];
     *reinterpret_cast<uint4 *>(&qw[4]) = q8[1];
     *reinterpret_cast<uint4 *>(&kw[0]) = k8[0];
     *reinterpret_cast<uint4 *>(&kw[4]) = k8[1];
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-        *reinterpret_cast<float4 *>(&a[4 * j]) = a4[j];
+    // the row group's 16 gates: lane l computes g of row 16 rg + (l mod 16) once, and every
+    // lane reads the value it needs from the lane of its half-warp that holds it (the same
+    // expf, so bit-identical).  At d = 128 a warp is one row group (both halves compute the
+    // same 16 values); at d = 64 each half-warp is one row group.
+    const int lane = tid & 31;
+    const float g_own = expf(p.log_g[row * D + 16 * rg + (lane & 15)]);
 
     float *st = p.state + ((int64_t)b * p.n_heads + h) * D * D;
     float4 S[16];
@@ -90,7 +91,7 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
     for (int r = 0; r < 16; ++r) {
-        const float g = expf(a[r]);
+        const float g = __shfl_sync(0xffffffffu, g_own, (lane & 16) | r);
         const float kk = (r & 1) ? bf16_hi(kw[r >> 1]) : bf16_lo(kw[r >> 1]);
         const float qq = (r & 1) ? bf16_hi(qw[r >> 1]) : bf16_lo(qw[r >> 1]);
         S[r].x = fmaf(g, S[r].x, kk * v4.x);
