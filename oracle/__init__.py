@@ -22,16 +22,26 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "hs_oracle.c")
 _LIB = os.path.join(_HERE, "liboracle.so")
+# a prebuilt oracle library to load instead (tests/test_oracle_mutants.py runs the pins
+# against deliberately broken copies of hs_oracle.c this way)
+_LIB_OVERRIDE = os.environ.get("HS_ORACLE_LIB")
 _lock = threading.Lock()
 _lib = None
 
 
+def compile_to(src: str, out: str) -> None:
+    """gcc -O2 of one oracle source into a shared library (no fast-math)."""
+    subprocess.run(["gcc", "-O2", "-fPIC", "-shared", "-std=c11", "-fno-fast-math",
+                    "-o", out, src, "-lm"], check=True)
+
+
 def build(force: bool = False) -> str:
     """Compile hs_oracle.c into liboracle.so (plain gcc, -O2, no fast-math)."""
+    if _LIB_OVERRIDE:
+        return _LIB_OVERRIDE
     if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
         tmp = _LIB + f".{os.getpid()}.tmp"
-        subprocess.run(["gcc", "-O2", "-fPIC", "-shared", "-std=c11", "-fno-fast-math",
-                        "-o", tmp, _SRC, "-lm"], check=True)
+        compile_to(_SRC, tmp)
         os.replace(tmp, _LIB)
     return _LIB
 
