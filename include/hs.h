@@ -321,8 +321,10 @@ typedef struct hs_linattn_shape {
  * log2-decay stays >= -10 in every key dimension and every operand provably fits
  * fp16; any other chunk runs on tf32 operands with the intra-chunk scores computed
  * in float32.  Against a float64 reference both stay within a max-normalised error
- * of 2e-3 per (problem, head) unless a head's largest output is one score q_i.k_j
- * whose terms cancel strongly, times a v_j far larger than the head's other values.
+ * of 2e-3 per (problem, head) unless one token's output exceeds every other output
+ * of its head by an order of magnitude or more (an outlier q, k or v on that token)
+ * and its dot products cancel strongly: the head's error is then that token's
+ * 11-bit operand rounding, amplified by the cancellation.
  * All of q, k, v, log_g, o, state must be 16-byte aligned.  q/k/v/log_g are only
  * read; o, state and the slots must not overlap the inputs or each other.
  * Token rows are 32-bit: b*max_tokens + n_tokens[b] must stay below 2^31.
