@@ -273,3 +273,22 @@ def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(mod, "_lib", None)
     with pytest.raises(RuntimeError):
         mod.hs_version()
+
+
+def test_c_client_compiles_links_and_runs(tmp_path):
+    """The public headers are C: a C11 client (tests/c_client/hs_client.c) compiles with
+    -Wall -Werror, links against libhs.so and runs its host-only checks."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no gcc")
+    cuda_inc = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "include")
+    exe = tmp_path / "hs_client"
+    libdir = os.path.dirname(hs.LIB_PATH)
+    subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-Werror", "-I", os.path.join(ROOT, "include"),
+                    "-I", cuda_inc, os.path.join(ROOT, "tests", "c_client", "hs_client.c"),
+                    "-o", str(exe), "-L", libdir, "-l:libhs.so", f"-Wl,-rpath,{libdir}"], check=True)
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0, r.stdout + r.stderr
+    assert "FAIL" not in r.stdout and r.stdout.count("ok ") >= 9
