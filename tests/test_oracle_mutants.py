@@ -44,8 +44,24 @@ MUTANTS = {
     "alignment ignores the hit": lambda s: s.replace("if (b > hit_len)\n            continue;", ""),
     "bf16 widened from the wrong bits": lambda s: s.replace("((uint32_t)b) << 16", "((uint32_t)b) << 15"),
     "state bytes counted in bf16": lambda s: s.replace("n_heads * d_k * d_v * 4", "n_heads * d_k * d_v * 2"),
+    "state bytes without the heads": lambda s: s.replace("n_lin_layers * n_heads * d_k * d_v * 4",
+                                                         "n_lin_layers * d_k * d_v * 4"),
     "scatter to the staging index": lambda s: s.replace(
         "memcpy(cache[l] + (int64_t)bt[j] * page_bytes,", "memcpy(cache[l] + (int64_t)j * page_bytes,"),
+    "gather from the staging index": lambda s: s.replace(
+        "cache[l] + (int64_t)bt[j] * page_bytes, (size_t)page_bytes);",
+        "cache[l] + (int64_t)j * page_bytes, (size_t)page_bytes);"),
+    "gather one page short": lambda s: s.replace(
+        "j < n_pages; ++j)\n            memcpy(staging", "j < n_pages - 1; ++j)\n            memcpy(staging"),
+    "slice ignores the column offset": lambda s: s.replace("+ r * row_bytes + col_off;", "+ r * row_bytes;"),
+    "slice of the first row only": lambda s: s.replace("+ r * row_bytes + col_off;", "+ col_off;"),
+    "slice direction swapped": lambda s: s.replace("if (gather)\n                    memcpy(s, c,",
+                                                   "if (!gather)\n                    memcpy(s, c,"),
+    "state copy from the first slot": lambda s: s.replace("memcpy(dst[i], src[i],", "memcpy(dst[i], src[0],"),
+    "state copy in reverse slot order": lambda s: s.replace("memcpy(dst[i], src[i],",
+                                                            "memcpy(dst[i], src[n - 1 - i],"),
+    "state copy of floats_each bytes": lambda s: s.replace("(size_t)floats_each * sizeof(float)",
+                                                           "(size_t)floats_each"),
 }
 
 

@@ -114,8 +114,17 @@ def test_restore_bytes_affine_and_table5_total():
     Bs = [oracle.align_prefix(N, N, list(range(C, N + 1, C)), 16)[0]
           for N, *_ in _rows("table4_alignment.txt")]
     assert 4 * sum(bytes_at(B) for B in Bs) == total
-    # and the state part scales with layers x heads x d_k x d_v x 4
-    assert oracle.restore_bytes(0, 0, 0, 3, 2, 8, 4) == 3 * 2 * 8 * 4 * 4
+
+
+def test_restore_bytes_of_the_workloads_derived_by_hand():
+    """Pages and float32 states of one resumed request, derived by hand from the workload
+    shapes in tests/golden/restore_bytes_configs.txt (the derivation is in its header): the
+    tiny stack's 12 pages of 8 KiB plus two 64 x 64 states, the hybrid and long-context
+    stacks at their longest prompts, and a states-only restore."""
+    rows = _rows("restore_bytes_configs.txt")
+    assert len(rows) == 4
+    for n_full, n_pages, page_bytes, n_lin, heads, dk, dv, total in rows:
+        assert oracle.restore_bytes(n_full, n_pages, page_bytes, n_lin, heads, dk, dv) == total
 
 
 # ---------------------------------------------------------------- recurrence
@@ -333,6 +342,54 @@ def test_rank_slices_reassemble_the_full_page_transfer():
             assert np.array_equal(a, b)
     for a, b in zip(got, want):
         assert np.array_equal(a, b)
+
+
+# float32 bit patterns a state restore must carry through unchanged: quiet and signalling
+# NaNs with payloads, both zeros, both infinities, the smallest and largest subnormals, the
+# largest normal, and ordinary values
+SPECIAL_F32 = np.array([0x7FC00000, 0xFFC12345, 0x7FA00001, 0xFF800001, 0x00000000, 0x80000000,
+                        0x7F800000, 0xFF800000, 0x00000001, 0x807FFFFF, 0x7F7FFFFF, 0x3F800000,
+                        0xC0490FDB, 0x00800000], np.uint32)
+
+
+def _slot_bits(n, floats_each, tag):
+    """n source slots whose words differ by slot and by position: the special patterns
+    first, then words that encode (tag, slot, index)."""
+    out = []
+    for i in range(n):
+        w = np.array([(tag << 24) ^ (i << 16) ^ x ^ 0x3C000000 for x in range(floats_each)],
+                     np.uint32)
+        m = min(len(SPECIAL_F32), floats_each)
+        w[:m] = np.roll(SPECIAL_F32, i)[:m]
+        out.append(w)
+    return out
+
+
+def test_copy_slots_bitwise_with_special_values():
+    """The state restore and the checkpoint writer (Section 1: a recurrent state updated in
+    place is restored, not recomputed; Section 2.2: the state at B) are copies of float32
+    slots: every bit pattern arrives unchanged in the slot of the same index, and the
+    destination past floats_each keeps its poison."""
+    n, fe, guard = 5, 37, 11
+    src_bits = _slot_bits(n, fe, 1)
+    src = [b.view(np.float32) for b in src_bits]
+    dst = [np.full(fe + guard, 0xDEADBEEF, np.uint32).view(np.float32) for _ in range(n)]
+    oracle.copy_slots(src, dst, fe)
+    for i in range(n):
+        got = dst[i].view(np.uint32)
+        assert np.array_equal(got[:fe], src_bits[i]), i
+        assert (got[fe:] == 0xDEADBEEF).all(), i
+    # the slots are distinct, so a copy from the wrong slot cannot pass the check above
+    assert len({b.tobytes() for b in src_bits}) == n
+
+
+def test_copy_slots_of_zero_slots_or_zero_floats_touch_nothing():
+    src = [b.view(np.float32) for b in _slot_bits(3, 8, 2)]
+    dst = [np.full(8, 0xDEADBEEF, np.uint32).view(np.float32) for _ in range(3)]
+    oracle.copy_slots(src, dst, 0)
+    oracle.copy_slots(src[:0], dst[:0], 8)
+    for d in dst:
+        assert (d.view(np.uint32) == 0xDEADBEEF).all()
 
 
 def test_bf16_rounding_is_round_to_nearest_even():
