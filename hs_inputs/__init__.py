@@ -213,3 +213,65 @@ SWEEP_LENGTHS = tuple(range(512, 4608 + 1, 512))      # nine prompt lengths
 LONG_LENGTHS = (16384, 32768, 65536)
 PARTIAL_HIT_SHORTFALL = 37                              # partial hit: hit = L - 37
 DECODE_STEPS = 64
+
+
+# ---------------------------------------------------------------------------
+# seeded stress calls (the accuracy campaign of the prefill kernels)
+# ---------------------------------------------------------------------------
+
+@dataclasses.dataclass
+class StressCase:
+    """One seeded random prefill call built to stress the kernels' numerics."""
+    seed: int
+    d: int
+    pos0: list
+    n_tokens: list
+    ckpt_interval: int
+    inputs: LinearInputs
+    S0: np.ndarray
+
+
+def _scaled_bf16(bits: np.ndarray, factor: float) -> np.ndarray:
+    return f32_to_bf16_bits(bf16_bits_to_f32(bits) * np.float32(factor))
+
+
+def gen_stress_case(seed: int) -> StressCase:
+    """Random batch (1-4 problems of 1-3 heads, d = 64 or 128), resume points in [0, 700),
+    tails of 0-1, 0-11 or 0-599 tokens, checkpoint interval 0/64/128/256/512, and up to
+    four random token ranges of one stress kind each: growing gates (+0.02), gates of -30
+    or -1.2, one zero gate (-1e4), v scaled by 2^17, or q and k scaled by 64; the starting
+    state N(0, 0.25) scaled by 1, 100 or 2^16."""
+    rng = np.random.default_rng(seed)
+    d = int(rng.choice([64, 128, 128, 128]))
+    B, nH = int(rng.integers(1, 5)), int(rng.integers(1, 4))
+    C = int(rng.choice([0, 64, 128, 256, 512]))
+    pos0 = [int(x) for x in rng.integers(0, 700, B)]
+    mode = int(rng.integers(4))
+    if mode == 0:
+        n_tok = [int(x) for x in rng.integers(0, 2, B)]
+    elif mode == 1:
+        n_tok = [int(x) for x in rng.integers(0, 12, B)]
+    else:
+        n_tok = [int(x) for x in rng.integers(0, 600, B)]
+    T = max(max(n_tok), 1)
+    inp = gen_linear(seed + 1000, 0, B, T, nH, d, d)
+    for _ in range(int(rng.integers(0, 5))):
+        b, t0 = int(rng.integers(B)), int(rng.integers(T))
+        ln = int(rng.integers(1, 70))
+        kind = int(rng.integers(6))
+        if kind == 0:
+            inp.a[b, t0:t0 + ln] = 0.02
+        elif kind == 1:
+            inp.a[b, t0:t0 + ln] = -30.0
+        elif kind == 2:
+            inp.a[b, t0] = -1e4
+        elif kind == 3:
+            inp.v[b, t0:t0 + ln] = _scaled_bf16(inp.v[b, t0:t0 + ln], 2.0 ** 17)
+        elif kind == 4:
+            inp.q[b, t0:t0 + ln] = _scaled_bf16(inp.q[b, t0:t0 + ln], 64.0)
+            inp.k[b, t0:t0 + ln] = _scaled_bf16(inp.k[b, t0:t0 + ln], 64.0)
+        else:
+            inp.a[b, t0:t0 + ln] = -1.2
+    S0 = gen_state(seed + 1000, 0, B, nH, d, d) * float(rng.choice([1.0, 1.0, 100.0, 2.0 ** 16]))
+    return StressCase(seed=seed, d=d, pos0=pos0, n_tokens=n_tok, ckpt_interval=C, inputs=inp,
+                      S0=S0.astype(np.float32))

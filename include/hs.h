@@ -320,11 +320,18 @@ typedef struct hs_linattn_shape {
  * bits, float32 accumulation and state) when its log-gates are <= 0, its total
  * log2-decay stays >= -10 in every key dimension and every operand provably fits
  * fp16; any other chunk runs on tf32 operands with the intra-chunk scores computed
- * in float32.  Against a float64 reference both stay within a max-normalised error
- * of 2e-3 per (problem, head) unless one token's output exceeds every other output
- * of its head by an order of magnitude or more (an outlier q, k or v on that token)
- * and its dot products cancel strongly: the head's error is then that token's
- * 11-bit operand rounding, amplified by the cancellation.
+ * in float32.  On both paths a token's own score A_ii = q_i . k_i is summed in
+ * float32 from the bf16 inputs, so operand rounding enters only through the
+ * products of different tokens and through the state.  Per output element,
+ * with eps = 2^-11 and Q~ = q 2^Lam, K~ = k 2^-Lam the decayed operands of the
+ * chunk, the error is at most about
+ *   2 eps (sum_d |Q~_id| |S_de| + sum_{j<i} |v_je| sum_d |Q~_id K~_jd|)
+ *     + eps sum_{j<=i} |A_ij| |v_je|
+ * plus the error the state carries in from earlier chunks (the same form).
+ * This stays below 2e-3 of the head's largest output whenever those sums of
+ * magnitudes are within about 1,000 times of it: over 3,000 seeded stress calls
+ * (tails up to 600 tokens, v scaled by 2^17, q and k by 64, gates of -30, -1.2,
+ * -1e4 and +0.02, states up to 2^16) the largest max-normalised error was 5.6e-4.
  * All of q, k, v, log_g, o, state must be 16-byte aligned.  q/k/v/log_g are only
  * read; o, state and the slots must not overlap the inputs or each other.
  * Token rows are 32-bit: b*max_tokens + n_tokens[b] must stay below 2^31.

@@ -75,6 +75,11 @@ constexpr float kLog2e = 1.4426950408889634f;
 // a gate of -1e4) for the differences Lam_i - Lam_j of later tokens to keep their precision.
 constexpr float kGateFloor = -100.0f;
 constexpr float kF16Lim = 32768.0f;         // fast-path fp16 operands stay below 2^15
+// a decision taken mid-run bounds the state it starts from (the measured |S| of the previous
+// segment's start plus that segment's largest update); the bound is scaled by this margin so
+// that whenever it passes, the measured state (what a run resumed at that segment checks)
+// passes too: rounding can put the computed state a few ulps above the exact-arithmetic bound
+constexpr float kBoundMargin = 1.00390625f; // 1 + 2^-8
 constexpr float kLamRange = 10.0f;          // fast path: a segment's total log2-decay >= -10, so
                                             // Q~ = q 2^Lam stays far from fp16's subnormals
 constexpr uint64_t kTimeoutNs = 1000000000ull;
@@ -99,7 +104,9 @@ constexpr uint32_t OFF_RED = 200704;    // per warp [8][8]: builders max |q|, fa
                                         //   max |v| (0..3); state warps max |S| (4)
 constexpr uint32_t OFF_BAR = 200960;    // 8 mbarriers
 constexpr uint32_t OFF_MISC = 201024;   // TMEM base address, abort flag, decision, run result
-constexpr uint32_t SMEM_BYTES = 201056 + 1024;
+constexpr uint32_t OFF_DG = 201088;     // diagonal of A in float32, two sets by segment parity:
+                                        //   [set][key-dim half][64 tokens] partial sums  1 KiB
+constexpr uint32_t SMEM_BYTES = 202112 + 1024;
 constexpr uint32_t STAGE_BYTES = 3 * 16384 + 32768;
 
 // tensor memory: D_O alternates between two buffers by chunk parity, placed on
@@ -177,6 +184,30 @@ __device__ __forceinline__ float warp_max(float v)
     for (int o = 16; o > 0; o >>= 1)
         v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
     return v;
+}
+
+// warp sums of eight per-lane values as a transposing butterfly: every lane returns the sum
+// over the warp's 32 lanes of value x = (lane >> 2) & 7, added in the same order in every
+// lane that holds it
+__device__ __forceinline__ float warp_sum8(const float (&v)[8], int lane)
+{
+    const bool h4 = (lane & 16) != 0, h3 = (lane & 8) != 0, h2 = (lane & 4) != 0;
+    float w[4], y[2];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const float send = h4 ? v[j] : v[j + 4];
+        w[j] = (h4 ? v[j + 4] : v[j]) + __shfl_xor_sync(0xffffffffu, send, 16);
+    }
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+        const float send = h3 ? w[j] : w[j + 2];
+        y[j] = (h3 ? w[j + 2] : w[j]) + __shfl_xor_sync(0xffffffffu, send, 8);
+    }
+    const float send = h2 ? y[0] : y[1];
+    float z = (h2 ? y[1] : y[0]) + __shfl_xor_sync(0xffffffffu, send, 4);
+    z += __shfl_xor_sync(0xffffffffu, z, 2);
+    z += __shfl_xor_sync(0xffffffffu, z, 1);
+    return z;
 }
 
 __device__ __forceinline__ float bf16f(uint16_t x)
@@ -262,7 +293,10 @@ __device__ __forceinline__ void zero_tail(uint8_t *smem, int L, bool builders_on
 // memory; 2^{Lam_last} into gam slot `gslot`) while it writes Q~ and K~ (token-major, the
 // d-contractions' operands) and K~^T (rows of [A ; K~^T]), fp16, with 4- and 16-byte
 // stores.  Then thread (e, half) packs V^T into TMEM.  Per warp: max |q|, |k|, |v| and
-// whether every operand fits fp16 (for the guard).
+// whether every operand fits fp16 (for the guard).  The diagonal A_ii = q_i . k_i (no decay
+// between a token and itself) is summed in float32 from the bf16 inputs, each warp's 64 key
+// dims by a butterfly, into the set's diagonal partials: fp16 Q~ and K~ would round the
+// terms of that dot product to 11 bits, which a token whose own q . k cancels cannot afford.
 __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, int par, int gslot)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -322,9 +356,11 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
     __half2 hq = __float2half2_rn(0.f), hk = hq;                 // max |Q~|, |K~| (fp16)
     // two groups of 8 tokens; within a group, token pairs: Q~ and K~ as fp16 pairs of key
     // dims, K~^T rows 2dp and 2dp+1 as fp16 pairs of tokens (byte permutes of the K~ pairs)
+    float *sDg = reinterpret_cast<float *>(smem + OFF_DG) + par * 128 + (warp & 1) * 64;
 #pragma unroll 1
     for (int grp = 0; grp < 2; ++grp) {
         uint32_t kt0[4], kt1[4];
+        float pd[8];   // q . k over this thread's two key dims, tokens 8 grp + 0..7 of its quarter
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             uint32_t kp[2];
@@ -340,6 +376,7 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
                 const float k0 = __uint_as_float(k2 << 16), k1 = __uint_as_float(k2 & 0xFFFF0000u);
                 const uint32_t qp = pack_h2(q0 * ex2(run0), q1 * ex2(run1));
                 kp[t] = pack_h2(k0 * ex2(-run0), k1 * ex2(-run1));
+                pd[2 * u + t] = fmaf(q1, k1, q0 * k0);
                 *reinterpret_cast<uint32_t *>(set + S_QH + h_off(64, i, 2 * dp)) = qp;
                 *reinterpret_cast<uint32_t *>(set + S_KH + h_off(64, i, 2 * dp)) = kp[t];
                 bq = bmax_abs(bq, q2);
@@ -351,6 +388,11 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
             kt1[u] = __byte_perm(kp[0], kp[1], 0x7632);   // key dim 2dp+1
         }
         const int j0 = 16 * qt + 8 * grp;
+        {
+            const float dsum = warp_sum8(pd, lane);
+            if ((lane & 3) == 0)
+                sDg[j0 + ((lane >> 2) & 7)] = dsum;
+        }
         *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowK + 2 * dp, j0)) =
             make_uint4(kt0[0], kt0[1], kt0[2], kt0[3]);
         *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowK + 2 * dp + 1, j0)) =
@@ -468,6 +510,9 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
     const int rowA = par ? 128 : 0;
     float r[32];
     tmem_ld32(tmem + lrow + (par ? TM_A1 : TM_A0) + jb, r);
+    // the diagonal from the builders' float32 partials (the two key-dim halves)
+    const float *sDg = reinterpret_cast<const float *>(smem + OFF_DG) + par * 128;
+    const float dg = (i >= jb && i < jb + 32) ? sDg[i] + sDg[64 + i] : 0.f;
     tmem_wait_ld();
     uint8_t *set = smem + par * SET_BYTES;
 #pragma unroll
@@ -476,7 +521,9 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             const int j0 = jb + 8 * c + 2 * u;
-            w[u] = pack_h2(j0 <= i ? r[8 * c + 2 * u] : 0.f, j0 + 1 <= i ? r[8 * c + 2 * u + 1] : 0.f);
+            const float x0 = j0 == i ? dg : (j0 <= i ? r[8 * c + 2 * u] : 0.f);
+            const float x1 = j0 + 1 == i ? dg : (j0 + 1 <= i ? r[8 * c + 2 * u + 1] : 0.f);
+            w[u] = pack_h2(x0, x1);
         }
         *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowA + i, jb + 8 * c)) =
             make_uint4(w[0], w[1], w[2], w[3]);
@@ -787,9 +834,10 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
 
     // the guard of a built fast segment (state warps, after the wait for the builders): log-gates
     // <= 0, and every fp16 operand (Q~, K~, V, A, the fp16 copy of the state it starts from)
-    // below 2^15 in magnitude
+    // below 2^15 in magnitude.  Returns whether the segment's own inputs pass; `state_ok` says
+    // whether the state (its measured magnitude, or a bound on it) passes too.
     float mk_new = 0.f, mv_new = 0.f;
-    auto guard = [&](float s_bound) -> bool {
+    auto guard = [&](float s_mag, bool &state_ok) -> bool {
         float mq = 0.f, mk = 0.f, mv = 0.f;
         bool ok = true;
 #pragma unroll
@@ -801,7 +849,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
         mk_new = mk;
         mv_new = mv;
-        return ok && 128.0f * mq * mk < kF16Lim && s_bound < kF16Lim;
+        state_ok = s_mag < kF16Lim;
+        return ok && 128.0f * mq * mk < kF16Lim;
     };
 
     // ---- one exact segment, from staged inputs, no decay pending and no MMA in flight;
@@ -959,8 +1008,12 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     //   bar_go:    state warps -> builders, the decision on segment k is made (sMisc[2]);
     //              when it is fast, it also means the operand set of segment k+1 is free
     //              (the products of segment k-1 are complete)
-    // A run ends after the last long segment or before a segment the guard sends to the
-    // exact path; the groups then meet CTA-wide.  No MMA is in flight at either end.
+    // A run ends after the last long segment, before a segment whose own inputs the guard
+    // sends to the exact path, or before a segment whose state bound fails: a decision inside a
+    // run only has a bound on the state it starts from (that state is still being computed), so
+    // such a segment starts a new run, whose first decision reads the measured state exactly as
+    // a run resumed from a checkpoint at that segment does.  The groups then meet CTA-wide.
+    // No MMA is in flight at either end.
     auto outp = [&](int64_t t) { return p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D; };
     int kseq = 0;   // long segments of the current run so far (slot of 2^{Lam_last}: kseq mod 4)
     auto builder_run = [&](int64_t rpos, int64_t rtok) {
@@ -1013,19 +1066,23 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     };
     auto state_run = [&](int64_t rpos, int64_t rtok) {
         int par = 0;
-        bool pend = false, stop_exact = false;
+        bool pend = false;
+        uint32_t stop = 0;   // why the run ended: 0 done or short segment, 1 exact, 2 new run
         int pend_par = 0, pend_L = 0, pend_g = 0;
         int64_t pend_tok = 0, pend_end = 0;
         float mk_cur = 0.f, mv_cur = 0.f;
         if (!wait_group(2, kIssuer, bar_built, ph_built))
             return;
-        bool fast = guard(state_max());
+        // first segment of a run: the measured state (float32 maximum of the last state pass
+        // or of the loaded state)
+        bool state_ok;
+        bool fast = guard(state_max(), state_ok) && state_ok;
         if (tid == kIssuer) {
             sMisc[2] = fast ? 1u : 0u;
             if (!fast)
                 mbar_arrive(bar_go);
         }
-        stop_exact = !fast;
+        stop = fast ? 0u : 1u;
         // a segment sent to the exact path: its (unused) D_A product is drained first
         if (!fast && !wait_group(2, kIssuer, bar_a, ph_a0))
             return;
@@ -1085,16 +1142,20 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             ++kseq;
             if (!is_long(rpos))
                 break;
-            // the builders' next segment, and the decision on it
+            // the builders' next segment, and the decision on it: the state it starts from is
+            // bounded by the fp16 copy's largest |S| at this segment's start plus this segment's
+            // largest update, 64 max|k| max|v| (the decay factors are <= 1)
             if (!wait_group(2, kIssuer, bar_built, ph_built))
                 return;
-            fast = guard(state_max() + 64.0f * mk_cur * mv_cur);
+            const bool inputs_ok =
+                guard((state_max() + 64.0f * mk_cur * mv_cur) * kBoundMargin, state_ok);
+            fast = inputs_ok && state_ok;
             if (tid == kIssuer) {
                 sMisc[2] = fast ? 1u : 0u;
                 if (!fast)
                     mbar_arrive(bar_go);
             }
-            stop_exact = !fast;
+            stop = fast ? 0u : (inputs_ok ? 2u : 1u);
             if (!fast && !(par ? wait_group(2, kIssuer, bar_a1, ph_a1) : wait_group(2, kIssuer, bar_a, ph_a0)))
                 return;
         }
@@ -1108,7 +1169,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 return;
         }
         if (tid == kIssuer) {
-            sMisc[3] = stop_exact ? 1u : 0u;
+            sMisc[3] = stop;
             sRun[0] = rpos;
             sRun[1] = rtok;
         }
@@ -1142,13 +1203,13 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (!sync_all())
             break;
         tc_fence_after();
-        const bool exact = sMisc[3] != 0;
+        const uint32_t stop = sMisc[3];
         pos = sRun[0];
         tok = sRun[1];
         kseq = 0;
-        if (exact) {
-            // the segment at pos takes the exact path: restage its inputs (the copy of the
-            // next segment may be in flight), then every thread runs it
+        if (stop != 0) {
+            // the segment at pos takes the exact path (1) or starts a new run (2): restage its
+            // inputs (the copy of the next segment may be in flight)
             const int Lx = seg_len(pos);
             if (tid == kLoader) {
                 if (tma_pending && !mbar_wait_bounded(bar_tma, ph_tma, kTimeoutNs))
@@ -1157,6 +1218,9 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     ph_tma ^= 1;
                 issue_tma(tok);
             }
+            if (stop == 2)
+                continue;   // the new run waits for the copy
+            // every thread runs the exact segment
             if (!wait_tma())
                 break;
             if (!exact_segment(tok, Lx, 0, 0, pos + Lx))

@@ -165,6 +165,57 @@ def test_fp16_range_guards_take_the_exact_path(case):
         assert np.array_equal(ck_r[0].view(np.uint32), cks[0][m + 1:].view(np.uint32))
 
 
+@pytest.mark.parametrize("kernel", [pytest.param(hs.HS_LINATTN_CHUNKED_TC, id="tc"),
+                                    pytest.param(hs.HS_LINATTN_AUTO, id="auto")])
+def test_state_bound_band_resumes_bitwise(kernel):
+    """A decision inside a fast run only has a bound on the state it starts from (the state
+    before the previous segment plus that segment's largest update).  Here the bound exceeds
+    the fp16 limit 2^15 while the state itself, halved by chunk 0's gates, stays far below it:
+    a full run from S0 must decide chunk 1 on the measured state, as a run resumed from the
+    checkpoint at 64 does, so the two agree bit for bit (and stay within 2e-3 of the oracle)."""
+    dev = device()
+    N, C, nH, d = 192, 64, 2, 128
+    inp = gen_linear(41, 0, 1, N, nH, d, d)
+    inp.a[0, :64] = np.float32(np.log(0.5) / 64)           # chunk 0 decays the state by 1/2
+    for x in (inp.k, inp.v):                                  # a large update in chunk 0
+        x[0, :64] = f32_to_bf16_bits(bf16_bits_to_f32(x[0, :64]) * np.float32(24.0))
+    S0 = gen_state(41, 0, 1, nH, d, d)
+    S0 = (S0 * np.float32(31000.0 / np.abs(S0).max())).astype(np.float32)
+    kb = np.abs(bf16_bits_to_f32(inp.k[0, :64])).max()
+    vb = np.abs(bf16_bits_to_f32(inp.v[0, :64])).max()
+    assert np.abs(S0).max() + 64 * kb * vb > 2.0 ** 15       # the bound fails ...
+    o_f, S_f, ck_f = run_prefill(inp, [0], [N], S0, C, dev, kernel)
+    assert np.abs(ck_f[0][0]).max() < 2.0 ** 14               # ... the state does not
+    sub = type(inp)(*(x[:, 64:N].copy() for x in (inp.q, inp.k, inp.v, inp.a)))
+    o_r, S_r, ck_r = run_prefill(sub, [64], [N - 64], ck_f[0][0][None], C, dev, kernel)
+    assert np.array_equal(o_r[0].view(np.uint32), o_f[0, 64:N].view(np.uint32))
+    assert np.array_equal(S_r.view(np.uint32), S_f.view(np.uint32))
+    assert np.array_equal(ck_r[0].view(np.uint32), ck_f[0][1:].view(np.uint32))
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], S0=S0, C_=C)
+    _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], "state-bound band")
+
+
+@pytest.mark.parametrize("kernel", [pytest.param(hs.HS_LINATTN_CHUNKED_TC, id="tc"),
+                                    pytest.param(hs.HS_LINATTN_AUTO, id="auto")])
+@pytest.mark.parametrize("seed", [3, 7, 9])
+def test_dominant_token_whose_own_score_cancels(kernel, seed):
+    """One token's q . k cancels to about 1 % of sum_d |q_d k_d| while its v, scaled by 2^17,
+    makes its output the head's largest by far: its error is the error of its own score
+    A_ii = q_i . k_i, which the fast path sums in float32 from the bf16 inputs (fp16 operands
+    would round each term to 11 bits and leave errors of up to 6.5e-3 here)."""
+    dev = device()
+    inp = gen_linear(seed, 0, 1, 64, 1, 128, 128)
+    q = bf16_bits_to_f32(inp.q[0, 63, 0]).astype(np.float64)
+    k = bf16_bits_to_f32(inp.k[0, 63, 0]).astype(np.float64)
+    k = k - (q @ k - 0.005) / (q @ q) * q
+    inp.k[0, 63, 0] = f32_to_bf16_bits(k.astype(np.float32))
+    inp.v[0, 63, 0] = f32_to_bf16_bits(bf16_bits_to_f32(inp.v[0, 63, 0]) * np.float32(2.0 ** 17))
+    o, S, cks = run_prefill(inp, [0], [64], None, 64, dev, kernel)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [64], C_=64)
+    assert np.abs(ro[0, 63]).max() > 30 * np.abs(ro[0, :63]).max()
+    _check(o, S, cks, ro, rS, rck, [0], [64], "cancelling score")
+
+
 @pytest.mark.parametrize("pattern", ["first", "middle_pair", "last", "all"])
 def test_exact_segments_at_run_boundaries(pattern):
     """Segments sent to the exact path (growing gates) where a run of fast segments
