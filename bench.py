@@ -21,9 +21,10 @@ timed on the host cores as a CPU baseline.
 ``--impl reference`` times the oracle itself (CPU) on a bounded sample of
 the same workload.
 
-``--case decode|prefill|kv|ckpt`` runs one small piece of the workload a few
-times and prints its CUDA-event times (no JSON): the cases the committed ncu
-captures under profiles/ were taken on.  ``--case long`` prints resumed vs
+``--case decode|prefill|kv|ckpt|sweep`` runs one small piece of the workload
+and prints its CUDA-event times: the cases the committed ncu captures under
+profiles/ were taken on (``--source-hashes`` prints the source hash each
+profiles/*.txt row is keyed on).  ``--case long`` prints resumed vs
 recomputed TTFT for the long-context stack (L = 16k/32k/64k, batch 4).
 """
 from __future__ import annotations
@@ -82,6 +83,49 @@ def kv_bytes(n_layers, n_pages, page_bytes):
 KERNEL_OF = {"decode": "gla_decode_kernel<128>", "prefill": "gla_chunked_tc_kernel",
              "restore": "restore_request_kernel"}
 
+# the source file of each kernel named in profiles/*.txt (a "kernel@workload" key names the
+# kernel before the "@")
+KERNEL_SRC = {"gla_decode_kernel": "gla_decode.cu", "gla_chunked_tc_kernel": "gla_chunked_tc.cu",
+              "gla_recurrent_kernel": "gla_recurrent.cu", "restore_request_kernel": "restore_request.cu",
+              "kv_scatter_kernel": "kv_scatter.cu", "kv_gather_kernel": "kv_scatter.cu",
+              "kv_slices_kernel": "kv_scatter.cu", "slot_copy_kernel": "slot_copy.cu"}
+DTYPE = "bf16 q/k/v, fp32 log-gates; fp16 (fast) or tf32 (exact) MMA operands, fp32 accumulate, state and outputs"
+
+
+def source_hash(kernel: str) -> str:
+    """First 12 hex digits of the SHA-256 of the kernel's source file, then the library's
+    internal headers and the public header (what its machine code depends on): a profile row
+    captured under another hash describes another kernel."""
+    import hashlib
+    name = kernel.split("@")[0].split("<")[0]
+    csrc = os.path.join(ROOT, "paper_2609_15030_gb300", "csrc")
+    files = [os.path.join(csrc, KERNEL_SRC[name])]
+    files += sorted(os.path.join(csrc, f) for f in os.listdir(csrc) if f.endswith(".cuh"))
+    files.append(os.path.join(ROOT, "include", "hs.h"))
+    h = hashlib.sha256()
+    for f in files:
+        h.update(open(f, "rb").read())
+    return h.hexdigest()[:12]
+
+
+def _profile_rows(fname, ncols):
+    """Rows `kernel v1 .. v_ncols source_hash capture ...` of a profiles/ table whose source
+    hash still matches the kernel's source; stale rows map to None."""
+    p = os.path.join(ROOT, "profiles", fname)
+    out = {}
+    if os.path.exists(p):
+        for line in open(p):
+            f = line.split()
+            if len(f) < ncols + 2 or line.startswith("#"):
+                continue
+            kern, vals, hsh = f[0], f[1:1 + ncols], f[1 + ncols]
+            try:
+                fresh = source_hash(kern) == hsh
+            except (KeyError, OSError):
+                fresh = False
+            out[kern] = (vals, f[2 + ncols] if len(f) > 2 + ncols else "") if fresh else None
+    return out
+
 
 def _nvtx(name: str):
     """An NVTX range around one section of the run (visible to ncu --nvtx and nsys);
@@ -96,28 +140,16 @@ def _nvtx(name: str):
 
 def _traffic():
     """DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) from the
-    committed ncu captures listed in profiles/dram_traffic.txt ("kernel bytes" lines)."""
-    p = os.path.join(ROOT, "profiles", "dram_traffic.txt")
-    out = {}
-    if os.path.exists(p):
-        for line in open(p):
-            f = line.split()
-            if len(f) >= 2 and not line.startswith("#"):
-                out[f[0]] = int(float(f[1]))
-    return out
+    committed ncu captures listed in profiles/dram_traffic.txt; None for a kernel whose
+    source changed since its capture (the row's source hash no longer matches)."""
+    return {k: (int(float(v[0][0])) if v else None) for k, v in _profile_rows("dram_traffic.txt", 1).items()}
 
 
 def _tensor_pipe():
     """Tensor-pipe utilisation (of active, of elapsed cycles) from the committed ncu captures
-    listed in profiles/tensor_pipe.txt."""
-    p = os.path.join(ROOT, "profiles", "tensor_pipe.txt")
-    out = {}
-    if os.path.exists(p):
-        for line in open(p):
-            f = line.split()
-            if len(f) >= 3 and not line.startswith("#"):
-                out[f[0]] = {"active": float(f[1]), "elapsed": float(f[2]), "source": "ncu " + f[3]}
-    return out
+    listed in profiles/tensor_pipe.txt; None for a kernel changed since its capture."""
+    return {k: ({"active": float(v[0][0]), "elapsed": float(v[0][1]), "source": "ncu " + v[1]}
+                if v else None) for k, v in _profile_rows("tensor_pipe.txt", 2).items()}
 
 
 # ---------------------------------------------------------------------------
@@ -796,6 +828,160 @@ def e2e_run(wl, steps, warmup):
             "ms_per_step": round(t * 1e3 / steps, 3)}
 
 
+def _l2_flush(torch, dev, buf=[]):
+    """Write 512 MiB (more than the 129 MB L2) so the next call reads its inputs from HBM."""
+    if not buf:
+        buf.append(torch.empty(512 * 2 ** 20, dtype=torch.uint8, device=dev))
+    buf[0].fill_(1)
+
+
+def sweep_run(dev, reps=10):
+    """Single-layer kernel sweep: one linear layer, 16 heads, d = 128, checkpoints every 512,
+    batch 1.  For each L in 512..4608: the resumed tail prefill (c = C floor((L-1)/C), 512
+    tokens from the state at c, emitting the checkpoint at L; the hit L-37 aligns to the same
+    c) and the recomputation of [0,L) from the zero state emitting every checkpoint.  Each
+    call is timed alone between CUDA events with L2 flushed before it; median of `reps`."""
+    import torch
+    import paper_2609_15030_gb300 as hs
+    from hs_inputs import SWEEP, torch_gen_linear
+    S = SWEEP
+    nH, d, C, Lmax = S.n_heads, S.d, S.ckpt, max(SWEEP_LENGTHS)
+    q, k, v, a = torch_gen_linear(11, 0, 1, Lmax, nH, d, dev)
+    o = torch.empty((1, Lmax, nH, d), device=dev)
+    state = torch.empty((1, nH, d, d), device=dev)
+    ck = torch.randn((1, nH, d, d), device=dev,
+                     generator=torch.Generator(device=dev).manual_seed(12)) * 0.5
+    slots = torch.empty((Lmax // C, nH, d, d), device=dev)
+    shape = hs.make_shape(1, nH, d, d, Lmax, hs.HS_LINATTN_AUTO)
+    stream = torch.cuda.current_stream(dev)
+    tb, tbf = nH * d * 2, nH * d * 4
+    peak = _peaks()[0]
+    tensor = _tensor_pipe()
+    rows = []
+    for L in SWEEP_LENGTHS:
+        c, _, tail = hs.hs_align_prefix(L, L, list(range(C, L + 1, C)), S.page)
+        c37, _, _ = hs.hs_align_prefix(L, L - 37, list(range(C, L + 1, C)), S.page)
+        nck_t = hs.hs_linattn_num_checkpoints([c], [tail], C)
+        tail_ptrs = hs.ptr_array([slots[i] for i in range(nck_t)], dev) if nck_t else None
+        rec_ptrs = hs.ptr_array([slots[i] for i in range(L // C)], dev)
+
+        def resume():
+            hs.hs_linattn_prefill_from_state(
+                shape, q.data_ptr() + c * tb, k.data_ptr() + c * tb, v.data_ptr() + c * tb,
+                a.data_ptr() + c * tbf, o.data_ptr() + c * tbf, state, [c], [tail], C, tail_ptrs,
+                None, stream.cuda_stream)
+
+        def recompute():
+            hs.hs_linattn_prefill_from_state(shape, q, k, v, a, o, state, [0], [L], C, rec_ptrs,
+                                             None, stream.cuda_stream)
+        res = {}
+        for nm, fn, init in (("tail", resume, lambda: state.copy_(ck)),
+                             ("recompute", recompute, lambda: state.zero_())):
+            ts = []
+            for i in range(reps + 2):
+                init()
+                _l2_flush(torch, dev)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+                torch.cuda.synchronize(dev)
+                if i >= 2:
+                    ts.append(e0.elapsed_time(e1) * 1e-3)
+            res[nm] = statistics.median(ts)
+        b_tail = gla_bytes(1, nH, d, tail, nck_t)
+        b_rec = gla_bytes(1, nH, d, L, L // C)
+        tp_t = tensor.get(f"gla_chunked_tc_kernel@sweep_tail_{L}")
+        tp_r = tensor.get(f"gla_chunked_tc_kernel@sweep_recompute_{L}")
+        rows.append({
+            "L": L, "c": c, "c_hit_L-37": c37, "tail": tail,
+            "tail_us": round(res["tail"] * 1e6, 2),
+            "tail_tokens_per_s": round(tail / res["tail"], 1),
+            "tail_hbm_frac": round(b_tail / res["tail"] / 1e9 / peak, 4),
+            "tail_tensor_pipe": tp_t["active"] if tp_t else None,
+            "recompute_us": round(res["recompute"] * 1e6, 2),
+            "recompute_tokens_per_s": round(L / res["recompute"], 1),
+            "recompute_hbm_frac": round(b_rec / res["recompute"] / 1e9 / peak, 4),
+            "recompute_tensor_pipe": tp_r["active"] if tp_r else None})
+    del q, k, v, a, o, slots
+    return {"workload": "single-layer sweep: 16 heads, d = 128, C = 512, batch 1, tails of 512 "
+                        "(complete hit and hit L-37 align to the same c)",
+            "timing": f"each call alone, L2 flushed before it, median of {reps}",
+            "tensor_pipe": "sm__pipe_tensor_cycles_active, % of active cycles, from the committed "
+                           "ncu capture of `bench.py --case sweep` (null when the kernel changed since)",
+            "rows": rows}
+
+
+def tiny_run(dev, reps=20):
+    """Tiny hybrid stack (1 linear layer: 2 heads, d = 64, C = 64; 1 full layer: 2 KV heads,
+    head_dim 64, page 16), seed 0, N = 256, complete hit -> c = 192: the resumed request
+    (alignment, restore of 12 KV pages and the state at 192, the 64-token tail) against the
+    recomputation of [0,256) (prefill from the zero state emitting every checkpoint and the KV
+    write of 16 pages).  Latency of each arm, host-launched, median of `reps`; the resumed
+    outputs and final state must equal the recomputation's bit for bit."""
+    import torch
+    import paper_2609_15030_gb300 as hs
+    from hs_inputs import TINY, gen_linear, gen_kv_pages, gen_block_table
+    S = TINY
+    N, C, P, nH, d = 256, S.ckpt, S.page, S.n_heads, S.d
+    c, n_pages, tail = hs.hs_align_prefix(N, N, list(range(C, N + 1, C)), P)
+    x = gen_linear(0, 0, 1, N, nH, d, d, gates=S.gates)
+    dv = lambda arr: torch.from_numpy(arr.view(np.int16) if arr.dtype == np.uint16 else arr).to(dev)
+    q, k, v, a = dv(x.q), dv(x.k), dv(x.v), dv(x.a)
+    pb = S.page_bytes
+    NB = 64
+    staging = torch.from_numpy(gen_kv_pages(0, 0, N // P, pb).reshape(-1)).to(dev)
+    cache = torch.zeros(NB * pb, dtype=torch.uint8, device=dev)
+    bt = torch.from_numpy(gen_block_table(0, 0, N // P, NB)).to(dev)
+    sp, cp = hs.ptr_array([staging], dev), hs.ptr_array([cache], dev)
+    o_rec = torch.empty((1, N, nH, d), device=dev)
+    o_res = torch.empty((1, N, nH, d), device=dev)
+    st_rec = torch.zeros((1, nH, d, d), device=dev)
+    live = torch.zeros((1, nH, d, d), device=dev)
+    slots = torch.empty((N // C, nH, d, d), device=dev)
+    slot_ptrs = hs.ptr_array([slots[i] for i in range(N // C)], dev)
+    last_ptr = hs.ptr_array([slots[N // C - 1]], dev)
+    src = hs.ptr_array([slots[c // C - 1]], dev)
+    dst = hs.ptr_array([live], dev)
+    shape = hs.make_shape(1, nH, d, d, N, hs.HS_LINATTN_AUTO)
+    tb, tbf = nH * d * 2, nH * d * 4
+    stream = torch.cuda.current_stream(dev)
+
+    def recompute():
+        st_rec.zero_()
+        hs.hs_linattn_prefill_from_state(shape, q, k, v, a, o_rec, st_rec, [0], [N], C, slot_ptrs,
+                                         None, stream.cuda_stream)
+        hs.hs_restore_kv_pages(sp, cp, 1, bt, N // P, pb, NB, None, stream.cuda_stream)
+
+    def resume():
+        cc, npg, tl = hs.hs_align_prefix(N, N, list(range(C, N + 1, C)), P)
+        hs.hs_restore_request(sp, cp, 1, bt, npg, pb, NB, src, dst, 1, nH * d * d, None,
+                              stream.cuda_stream)
+        hs.hs_linattn_prefill_from_state(
+            shape, q.data_ptr() + cc * tb, k.data_ptr() + cc * tb, v.data_ptr() + cc * tb,
+            a.data_ptr() + cc * tbf, o_res.data_ptr() + cc * tbf, live, [cc], [tl], C, last_ptr,
+            None, stream.cuda_stream)
+    out = {}
+    for nm, fn in (("recompute", recompute), ("resume", resume)):
+        ts = []
+        for i in range(reps + 3):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            if i >= 3:
+                ts.append(e0.elapsed_time(e1) * 1e3)
+        out[nm + "_us"] = round(statistics.median(ts), 2)
+    same = (torch.equal(o_res[:, c:].view(torch.int32), o_rec[:, c:].view(torch.int32))
+            and torch.equal(live.view(torch.int32), st_rec.view(torch.int32)))
+    out.update({"N": N, "c": c, "pages": n_pages, "tail": tail, "resume_equals_recompute": bool(same),
+                "timing": f"host-launched calls between CUDA events, median of {reps}"})
+    return out
+
+
 # ---------------------------------------------------------------------------
 # the oracle on the host cores (CPU baseline / reference arm)
 # ---------------------------------------------------------------------------
@@ -862,6 +1048,107 @@ def cpu_baseline():
                       f"float64 token by token; {t:.1f} s wall on {cores} threads",
             "one_thread": {"value": round(toks1 / t1, 2), "unit": "tokens/s", "cores": 1,
                            "sample": f"request 0 of the same step (L = 512) on one thread, {t1:.1f} s wall"}}
+
+
+def cpu_baseline_configs():
+    """The float64 oracle as it stands on the host cores, on the other configurations:
+    the tiny stack's resumed request (in full), the sweep's nine tails and nine
+    recomputations (in full), one KV-stress request's page scatter (in full), and one
+    long-context request at L = 65,536: its page scatter and state copy in full, its
+    linear-attention work on one (layer, head) and scaled to all 18 x 32 heads of one request
+    (labelled extrapolated)."""
+    import oracle
+    from hs_inputs import SWEEP, TINY, LONG24, LONG_LENGTHS, gen_linear, gen_kv_pages, gen_block_table
+    cores = _cores()
+    out = {"cores": cores, "kind": "oracle"}
+    # tiny stack, one resumed request
+    S = TINY
+    N, C = 256, S.ckpt
+    x = gen_linear(0, 0, 1, N, S.n_heads, S.d, S.d, gates=S.gates)
+    stg = [gen_kv_pages(0, 0, N // S.page, S.page_bytes).reshape(-1)]
+    cache = [np.zeros(64 * S.page_bytes, np.uint8)]
+    bt = gen_block_table(0, 0, N // S.page, 64)
+    ck = [np.random.default_rng(1).standard_normal(S.n_heads * S.d * S.d).astype(np.float32)]
+    live = [np.zeros_like(ck[0])]
+    reps = 20
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        c, npg, tail = oracle.align_prefix(N, N, list(range(C, N + 1, C)), S.page)
+        oracle.scatter_pages(stg, cache, bt, npg, S.page_bytes)
+        oracle.copy_slots(ck, live, S.n_heads * S.d * S.d)
+        oracle.gla(x.q[:, c:], x.k[:, c:], x.v[:, c:], x.a[:, c:], [c], [tail],
+                   S0=live[0].reshape(1, S.n_heads, S.d, S.d), C_=C, threads=1)
+    t = (time.perf_counter() - t0) / reps
+    out["tiny"] = {"resume_us": round(t * 1e6, 1), "cores": 1,
+                   "sample": f"align + 12-page scatter + state copy + 64-token tail (2 heads, d = 64), "
+                             f"one thread, mean of {reps}"}
+    # sweep: the nine tails and recomputations, 16 heads in parallel
+    S = SWEEP
+    Lmax = max(SWEEP_LENGTHS)
+    x = gen_linear(11, 0, 1, Lmax, S.n_heads, S.d, S.d)
+    S0 = np.random.default_rng(12).standard_normal((1, S.n_heads, S.d, S.d)).astype(np.float32)
+    t_tail = t_rec = 0.0
+    for L in SWEEP_LENGTHS:
+        c = S.ckpt * ((L - 1) // S.ckpt)
+        t0 = time.perf_counter()
+        oracle.gla(x.q[:, c:L], x.k[:, c:L], x.v[:, c:L], x.a[:, c:L], [c], [L - c], S0=S0,
+                   C_=S.ckpt, threads=cores)
+        t_tail += time.perf_counter() - t0
+        t0 = time.perf_counter()
+        oracle.gla(x.q[:, :L], x.k[:, :L], x.v[:, :L], x.a[:, :L], [0], [L], C_=S.ckpt, threads=cores)
+        t_rec += time.perf_counter() - t0
+    n_tail = sum(L - S.ckpt * ((L - 1) // S.ckpt) for L in SWEEP_LENGTHS)
+    out["sweep"] = {"tail_tokens_per_s": round(n_tail / t_tail, 1),
+                    "recompute_tokens_per_s": round(sum(SWEEP_LENGTHS) / t_rec, 1), "cores": cores,
+                    "sample": f"all nine 512-token tails and recomputations of [0,L), 16 heads on "
+                              f"{cores} threads, {t_tail + t_rec:.1f} s wall"}
+    # KV stress: one request's scatter (48 layers x 256 pages x 64 KiB)
+    P = KVSTRESS.page_bytes
+    nL, npg = KVSTRESS.n_full, 4096 // KVSTRESS.page
+    stg = [np.ones(npg * P, np.uint8) for _ in range(nL)]
+    cache = [np.full(2 * npg * P, 0, np.uint8) for _ in range(nL)]   # touched before timing
+    bt = gen_block_table(40, 0, npg, 2 * npg)
+    oracle.scatter_pages(stg, cache, bt, npg, P)
+    t0 = time.perf_counter()
+    oracle.scatter_pages(stg, cache, bt, npg, P)
+    t = time.perf_counter() - t0
+    out["kv_stress"] = {"gbs": round(kv_bytes(nL, npg, P) / t / 1e9, 2), "cores": 1,
+                        "sample": "one request: 48 layers x 256 pages x 64 KiB (read + write bytes), "
+                                  f"one thread, {t:.2f} s"}
+    del stg, cache
+    # long context: one request at L = 65,536 (complete hit, c = 65,024)
+    S = LONG24
+    L = max(LONG_LENGTHS)
+    c = S.ckpt * ((L - 1) // S.ckpt)
+    npg = c // S.page
+    stg = [np.ones(npg * S.page_bytes, np.uint8) for _ in range(S.n_full)]
+    cache = [np.full(npg * S.page_bytes, 0, np.uint8) for _ in range(S.n_full)]
+    bt = np.arange(npg, dtype=np.int32)[::-1].copy()
+    ckl = [np.ones(S.n_heads * S.d * S.d, np.float32) for _ in range(S.n_lin)]
+    livel = [np.zeros_like(z) for z in ckl]
+    t0 = time.perf_counter()
+    oracle.scatter_pages(stg, cache, bt, npg, S.page_bytes)
+    oracle.copy_slots(ckl, livel, S.n_heads * S.d * S.d)
+    t_copy = time.perf_counter() - t0
+    del stg, cache
+    xl = gen_linear(13, 0, 1, 4096, 1, S.d, S.d)
+    t0 = time.perf_counter()
+    oracle.gla(xl.q[:, :L - c], xl.k[:, :L - c], xl.v[:, :L - c], xl.a[:, :L - c], [c], [L - c],
+               S0=None, C_=S.ckpt, threads=1)
+    t_head_tail = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    oracle.gla(xl.q, xl.k, xl.v, xl.a, [0], [4096], C_=S.ckpt, threads=1)
+    t_head_4k = time.perf_counter() - t0
+    heads = S.n_lin * S.n_heads
+    out["long"] = {
+        "L": L, "c": c, "extrapolated": True, "cores": 1,
+        "ttft_resume_s": round(t_copy + heads * t_head_tail, 2),
+        "ttft_recompute_s": round(heads * t_head_4k * L / 4096, 1),
+        "sample": f"one request of the batch of 4: page scatter of 6 layers x {npg} pages x 128 KiB and "
+                  f"18 state copies in full ({t_copy:.2f} s); the 512-token tail of one (layer, head) "
+                  f"({t_head_tail:.2f} s) x 576 heads; the recomputation from one head's first 4,096 "
+                  f"tokens ({t_head_4k:.2f} s) x 576 heads x L/4096; one thread"}
+    return out
 
 
 def run_reference(args):
@@ -959,6 +1246,12 @@ def run_case(name: str, iters: int = 5):
     elif name == "long":
         run_long(dev)
         return 0
+    elif name == "sweep":
+        # single-layer sweep: each L's 512-token tail from c, then its recomputation of [0,L),
+        # one call each with L2 flushed before it (18 prefill launches, L = 512 .. 4608)
+        r = sweep_run(dev, reps=1)
+        for row in r["rows"]:
+            print(json.dumps({k: row[k] for k in ("L", "tail_us", "recompute_us")}), flush=True)
     else:
         raise SystemExit(f"unknown case {name}")
     return 0
@@ -1043,9 +1336,18 @@ def run_long(dev, reps=3, quiet=False):
                     torch.cuda.synchronize(dev)
                     ts.append(e0.elapsed_time(e1))
                 res[nm] = statistics.median(ts)
+            # algorithmic bytes of each arm: resume = KV restore of [0,c) + state restore +
+            # the tail prefill of every linear layer; recompute = the prefill of [0,L) of every
+            # linear layer emitting every checkpoint + the KV write of L tokens
+            b_res = (B * kv_bytes(nF, n_pages, pb) + 2 * nL * B * nH * d * d * 4
+                     + nL * gla_bytes(B, nH, d, tail, 1 if L % C == 0 else 0))
+            b_rec = nL * gla_bytes(B, nH, d, L, L // C) + B * kv_bytes(nF, L // P, pb)
+            peak = _peaks()[0]
             row = {"L": L, "hit": hit, "c": c, "tail": tail, "ttft_resume_ms": round(res["resume"], 3),
                    "ttft_recompute_ms": round(res["recompute"], 3),
-                   "ratio": round(res["recompute"] / res["resume"], 1)}
+                   "ratio": round(res["recompute"] / res["resume"], 1),
+                   "resume_hbm_frac": round(b_res / (res["resume"] * 1e-3) / 1e9 / peak, 3),
+                   "recompute_hbm_frac": round(b_rec / (res["recompute"] * 1e-3) / 1e9 / peak, 3)}
             rows.append(row)
             if not quiet:
                 print(json.dumps(row), flush=True)
@@ -1095,9 +1397,15 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true",
                     help="skip TTFT arms, KV stress, e2e and CPU baseline")
-    ap.add_argument("--case", choices=["decode", "prefill", "kv", "ckpt", "long"],
+    ap.add_argument("--case", choices=["decode", "prefill", "kv", "ckpt", "long", "sweep"],
                     help="run one small standalone case for a profiler capture")
+    ap.add_argument("--source-hashes", action="store_true",
+                    help="print each profiled kernel's source hash (the key of profiles/*.txt rows)")
     args = ap.parse_args()
+    if args.source_hashes:
+        for k in sorted(KERNEL_SRC):
+            print(k, source_hash(k))
+        return 0
     if args.case:
         return run_case(args.case)
     if args.impl == "reference":
@@ -1178,13 +1486,14 @@ def main():
              "share_of_step": round(ms * 1e-3 / t_phases, 3)}
         if kern in tensor:
             r["tensor_pipe_frac"] = tensor[kern]
+        r["source_hash"] = source_hash(kern)
         return r
 
     dominant = max(groups, key=lambda k: groups[k][1])
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(t * 1e3 / args.steps, 3),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": DTYPE,
         "data": "synthetic",
         "config": {"workload": WORKLOAD, "tokens_per_step": TOKENS_PER_STEP,
                    "l2": "inputs larger than L2: four seeds x nine requests rotate "
@@ -1205,6 +1514,10 @@ def main():
         out["e2e"]["ms_per_step"] = wl_e2e["ms_per_step"]
         with _nvtx("ttft resume vs recompute"):
             out["ttft_us"] = ttft_arms(wl)
+        with _nvtx("tiny stack latency"):
+            out["tiny_latency"] = tiny_run(dev)
+        with _nvtx("single-layer sweep"):
+            out["sweep"] = sweep_run(dev)
         red = [1.0 - r["resume_us"] / r["recompute_us"] for r in out["ttft_us"].values()]
         out["paper_context"] = {
             "ttft_reduction": "46-64 %", "total_time_reduction": "1.9-7.0 %",
@@ -1239,6 +1552,7 @@ def main():
             out["ttft_long_ms"] = run_long(dev, quiet=True)
         with _nvtx("oracle baseline"):
             out["cpu_baseline"] = cpu_baseline()
+            out["cpu_baseline_configs"] = cpu_baseline_configs()
     if rank == 0:
         print(json.dumps(out))
     if ws > 1:
