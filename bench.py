@@ -670,6 +670,66 @@ def kv_host(dev, save=False, n_requests=8, pool=2):
     return out
 
 
+def host_link(dev, nbytes=1 << 30, reps=5):
+    """The host link's copy rate (NVLink-C2C between Grace memory and HBM) with the copy
+    engines: one 1 GiB transfer between pinned host memory and the device in each direction,
+    the same bytes as four concurrent 256 MiB transfers on four streams, and both directions
+    at once (1 GiB each way on two streams); medians of `reps`, CUDA events."""
+    import torch
+    host = [torch.empty(nbytes, dtype=torch.uint8).pin_memory() for _ in range(2)]
+    devb = [torch.empty(nbytes, dtype=torch.uint8, device=dev) for _ in range(2)]
+    host[0].fill_(1)
+    devb[0].fill_(2)
+    main = torch.cuda.current_stream(dev)
+    streams = [torch.cuda.Stream(dev) for _ in range(4)]
+
+    def timed(fn):
+        ts = []
+        for _ in range(reps + 1):
+            torch.cuda.synchronize(dev)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(main)
+            fn()
+            e1.record(main)
+            torch.cuda.synchronize(dev)
+            ts.append(e0.elapsed_time(e1) * 1e-3)
+        return statistics.median(ts[1:])
+
+    def split(dst, src):
+        q = nbytes // 4
+        for i, st in enumerate(streams):
+            st.wait_stream(main)
+            with torch.cuda.stream(st):
+                dst[i * q:(i + 1) * q].copy_(src[i * q:(i + 1) * q], non_blocking=True)
+        for st in streams:
+            main.wait_stream(st)
+
+    def both():
+        for st in streams[:2]:
+            st.wait_stream(main)
+        with torch.cuda.stream(streams[0]):
+            devb[1].copy_(host[0], non_blocking=True)
+        with torch.cuda.stream(streams[1]):
+            host[1].copy_(devb[0], non_blocking=True)
+        for st in streams[:2]:
+            main.wait_stream(st)
+    h2d = nbytes / timed(lambda: devb[1].copy_(host[0], non_blocking=True)) / 1e9
+    d2h = nbytes / timed(lambda: host[1].copy_(devb[0], non_blocking=True)) / 1e9
+    h2d4 = nbytes / timed(lambda: split(devb[1], host[0])) / 1e9
+    d2h4 = nbytes / timed(lambda: split(host[1], devb[0])) / 1e9
+    bi = 2 * nbytes / timed(both) / 1e9
+    del host, devb
+    torch.cuda.empty_cache()
+    return {"h2d_gbs": round(max(h2d, h2d4), 1), "d2h_gbs": round(max(d2h, d2h4), 1),
+            "bidirectional_gbs": round(bi, 1),
+            "h2d_one_copy_gbs": round(h2d, 1), "h2d_four_streams_gbs": round(h2d4, 1),
+            "d2h_one_copy_gbs": round(d2h, 1), "d2h_four_streams_gbs": round(d2h4, 1),
+            "method": "copy-engine transfers between 1 GiB pinned host buffers and HBM: one copy, "
+                      "four concurrent 256 MiB copies on four streams (the better of the two is the "
+                      "direction's peak), and 1 GiB each way at once; medians of 5, CUDA events"}
+
+
 def state_copy(dev, reps=20, pool=8):
     """The standalone checkpoint writer (hs_checkpoint_states; hs_restore_state is the same
     copy the other way) on the long-context stack's live states: 4 requests x 18 linear
@@ -1536,8 +1596,14 @@ def main():
         kv["traffic"] = _traffic().get("kv_scatter_kernel@kvstress")
         out["kv_restore"] = kv
         with _nvtx("kv host staging"):
+            link = host_link(dev)
+            out["host_link"] = link
             out["kv_restore_from_host"] = kv_host(dev)
             out["kv_save_to_host"] = kv_host(dev, save=True)
+            out["kv_restore_from_host"]["frac_of_link_h2d"] = round(
+                out["kv_restore_from_host"]["host_read_gbs"] / link["h2d_gbs"], 3)
+            out["kv_save_to_host"]["frac_of_link_d2h"] = round(
+                out["kv_save_to_host"]["host_write_gbs"] / link["d2h_gbs"], 3)
         with _nvtx("kv rank slices"):
             sl = kv_rank_slices(dev)
         sl["frac"] = round(sl["gbs"] / peak, 4)
