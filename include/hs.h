@@ -250,16 +250,16 @@ hs_status hs_checkpoint_states(const float *const *live_states, float *const *ck
 
 /* Which kernel hs_linattn_prefill_from_state runs. */
 typedef enum hs_linattn_kernel {
-    HS_LINATTN_AUTO = 0,       /* chunked tensor-core kernel when d_k == d_v == 128,
-                                  batch*max_tokens < 2^31 and some n_tokens exceeds
+    HS_LINATTN_AUTO = 0,       /* chunked tensor-core kernel when some n_tokens exceeds
                                   HS_SHORT_SEGMENT; the single-token kernel when every
                                   n_tokens is at most 1 (decode steps); else the recurrent
                                   kernel.  All three compute segments of at most
                                   HS_SHORT_SEGMENT tokens identically, so AUTO never changes
                                   results */
     HS_LINATTN_RECURRENT = 1,  /* per-token recurrence, CUDA cores */
-    HS_LINATTN_CHUNKED_TC = 2, /* chunked form on tcgen05 tensor cores (d_k == d_v == 128;
-                                  HS_ERR_UNSUPPORTED otherwise) */
+    HS_LINATTN_CHUNKED_TC = 2, /* chunked form on tcgen05 tensor cores (d_k == d_v, 64 or
+                                  128; at 64 the M = 128 products leave half their TMEM lanes
+                                  unused) */
     HS_LINATTN_SINGLE_TOKEN = 3 /* one decode step per problem, state in registers, no
                                   shared memory (HS_ERR_UNSUPPORTED if some n_tokens > 1) */
 } hs_linattn_kernel;

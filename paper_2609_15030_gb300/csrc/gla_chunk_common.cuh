@@ -22,7 +22,6 @@ namespace gck {
 
 using namespace ptx;
 
-constexpr int D = 128;    // d_k = d_v
 constexpr int CH = 64;    // chunk length (absolute grid)
 constexpr int NB = 256;   // operand builders (warps 0..7): cumulative gates, Q~, K~, K~^T, V^T
 constexpr int NW = 256;   // state warps (warps 8..15): state passes, masks, epilogues
@@ -47,21 +46,22 @@ constexpr float kLamRange = 10.0f;          // fast path: a segment's total log2
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr int kPrefetch = 2;                // segments requested into L2 ahead of the staged one
 
-// shared memory map (offsets from a 1024-byte aligned base).  Operands are
+// shared memory map (offsets from a 1024-byte aligned base), sized for the head width
+// D = d_k = d_v = 128 (a D = 64 head uses the first part of each region).  Operands are
 // K-major with the 128-byte swizzle.
 constexpr uint32_t SET_BYTES = 57344;   // one fast operand set:
-constexpr uint32_t S_QH = 0;            //   Q~  fp16 [64 tok i][128 d]                 16 KiB
-constexpr uint32_t S_KH = 16384;        //   K~  fp16 [64 tok j][128 d]                 16 KiB
-constexpr uint32_t S_B2H = 32768;       //   [A ; K~^T] fp16 [64 i + 128 d][64 tok j]   24 KiB
-constexpr uint32_t X_QT = 0;            // exact path (over both sets): Q~ tf32 [64][128]     32 KiB
-constexpr uint32_t X_LAM = 32768;       //   Lam f32 [64 tok][128 d], row-major                 32 KiB
-constexpr uint32_t X_B2 = 65536;        //   [A ; K^^T] tf32 [64 i + 128 d][64 tok j]           48 KiB
-constexpr uint32_t OFF_SQ = 114688;     // staged q  bf16 [64][128]                16 KiB
+constexpr uint32_t S_QH = 0;            //   Q~  fp16 [64 tok i][D]                     16 KiB
+constexpr uint32_t S_KH = 16384;        //   K~  fp16 [64 tok j][D]                     16 KiB
+constexpr uint32_t S_B2H = 32768;       //   [A ; K~^T] fp16 [64 i + D][64 tok j]       24 KiB
+constexpr uint32_t X_QT = 0;            // exact path (over both sets): Q~ tf32 [64][D]         32 KiB
+constexpr uint32_t X_LAM = 32768;       //   Lam f32 [64 tok][D], row-major                     32 KiB
+constexpr uint32_t X_B2 = 65536;        //   [A ; K^^T] tf32 [64 i + D][64 tok j]               48 KiB
+constexpr uint32_t OFF_SQ = 114688;     // staged q  bf16 [64][D]                  16 KiB
 constexpr uint32_t OFF_SK = 131072;     // staged k                                 16 KiB
 constexpr uint32_t OFF_SV = 147456;     // staged v                                 16 KiB
-constexpr uint32_t OFF_SG = 163840;     // staged log-gates f32 [64][128]           32 KiB
+constexpr uint32_t OFF_SG = 163840;     // staged log-gates f32 [64][D]             32 KiB
 constexpr uint32_t OFF_GAM = 196608;    // 2^{Lam_last} per key dim, four slots by chunk number   2 KiB
-constexpr uint32_t OFF_TOT = 198656;    // partial log2-decay totals [4 token quarters][128]  2 KiB
+constexpr uint32_t OFF_TOT = 198656;    // partial log2-decay totals [token groups][D]        2 KiB
 constexpr uint32_t OFF_RED = 200704;    // per warp [8][8]: builders max |q|, fast-path flag, max |k|,
                                         //   max |v| (0..3); state warps max |S| (4)
 constexpr uint32_t OFF_BAR = 200960;    // 8 mbarriers
@@ -69,30 +69,44 @@ constexpr uint32_t OFF_MISC = 201024;   // TMEM base address, abort flag, decisi
 constexpr uint32_t OFF_DG = 201088;     // diagonal of A in float32, two sets by segment parity:
                                         //   [set][key-dim half][64 tokens] partial sums  1 KiB
 constexpr uint32_t SMEM_BYTES = 202112 + 1024;
-constexpr uint32_t STAGE_BYTES = 3 * 16384 + 32768;
 
 // tensor memory: D_O alternates between two buffers by chunk parity, placed on
-// either side of S^T so that [D_O0 | S^T] and [S^T | D_O1] are each one N=192
-// accumulator; even chunks order the 192-row operand as [A ; K~^T], odd ones
-// as [K~^T ; A].
+// either side of S^T so that [D_O0 | S^T] and [S^T | D_O1] are each one accumulator of
+// N = 64 + D; even chunks order the (64 + D)-row operand as [A ; K~^T], odd ones as
+// [K~^T ; A].  Every MMA has M = 128 (TMEM lanes = value dim e, or query row i for D_A):
+// with D = 64 the lanes 64..127 of the state-side products are computed and never read.
 constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t TM_O0 = 0;           // D_O of even chunks (lane e, col i), 64 cols
-constexpr uint32_t TM_S = 64;           // S^T  float32, 128 lanes x 128 cols
-constexpr uint32_t TM_O1 = 192;         // D_O of odd chunks
-constexpr uint32_t TM_SH = 256;         // S^T fp16 copy, two key dims per column      64 cols
+constexpr uint32_t TM_S = 64;           // S^T  float32, 128 lanes x D cols
+constexpr uint32_t TM_SH = 256;         // S^T fp16 copy, two key dims per column      D/2 cols
 constexpr uint32_t TM_A0 = 320;         // D_A of even segments, 128 lanes x 64 cols (lanes 0..63 used)
 constexpr uint32_t TM_V = 384;          // V^T: fast, fp16 pairs 2 x 32 cols; exact, f32 64 cols
 constexpr uint32_t TM_A1 = 448;         // D_A of odd segments
-// exact path (no fast-path data live): S^T as two tf32 parts for S^T Q~^T, hi in the 128
-// columns of D_O1 and the fp16 copy, lo in the two D_A buffers (key dims 0..63, 64..127)
-constexpr uint32_t TM_SHI = 192;
+// exact path (no fast-path data live): S^T as two tf32 parts for S^T Q~^T, hi in the D
+// columns right of S^T (D_O1 and, for D = 128, the fp16 copy), lo in the D_A buffers (key
+// dims 0..63, 64..127)
 constexpr uint32_t TM_SLO0 = 320;
 constexpr uint32_t TM_SLO1 = 448;
 
 constexpr uint32_t IDF_N64 = idesc_f16(128, 64);
-constexpr uint32_t IDF_N192 = idesc_f16(128, 192);
 constexpr uint32_t IDT_N64 = idesc_tf32(128, 64, 0, 0);
-constexpr uint32_t IDT_N128 = idesc_tf32(128, 128, 0, 0);
+
+// what depends on the head width D (64 or 128)
+template <int D>
+struct Geo {
+    static_assert(D == 64 || D == 128, "head width");
+    static constexpr int DP = D / 2;              // builder threads per token group (key-dim pairs)
+    static constexpr int NQ = NB / DP;            // token groups of the build: 4 or 8
+    static constexpr int TPG = CH / NQ;           // tokens per group: 16 or 8
+    static constexpr int CW = D / 2;              // state columns per state thread: 64 or 32
+    static constexpr int NG = D / 16;             // short segments: partial sums over 16 key rows
+    static constexpr int ROWS = 64 + D;           // rows of the [A ; K~^T] operands
+    static constexpr uint32_t O1 = TM_S + D;      // D_O of odd chunks, right of S^T
+    static constexpr uint32_t SHI = TM_S + D;     // exact path: hi part of S^T
+    static constexpr uint32_t IDF_UPD = idesc_f16(128, 64 + D);    // [D_O | S^T] += V^T [..]^T
+    static constexpr uint32_t IDT_ST = idesc_tf32(128, D, 0, 0);   // exact: S^T += V^T K^
+    static constexpr uint32_t STAGE = 3 * CH * D * 2 + CH * D * 4;  // staged q, k, v, log-gates
+};
 
 struct TmaMaps {
     CUtensorMap q, k, v, g;
@@ -222,23 +236,25 @@ __device__ __forceinline__ float rna_tf32(float x)
 
 // zero the staged rows past a segment of L < 64 tokens (all threads, or the builder
 // warps only)
+template <int D>
 __device__ __forceinline__ void zero_tail(uint8_t *smem, int L, bool builders_only)
 {
     const int tid = threadIdx.x;
+    constexpr int QV = D / 8, RV = 5 * D / 8;   // 16-byte vectors per q/k/v row, per token
 
     if (L < CH) {
         const int nthr = builders_only ? NB : NT;
-        for (int idx = tid; idx < (CH - L) * 80; idx += nthr) {
-            const int row = L + idx / 80, c = idx % 80;
+        for (int idx = tid; idx < (CH - L) * RV; idx += nthr) {
+            const int row = L + idx / RV, c = idx % RV;
             uint4 *dst;
-            if (c < 16)
-                dst = reinterpret_cast<uint4 *>(smem + OFF_SQ + row * 256) + c;
-            else if (c < 32)
-                dst = reinterpret_cast<uint4 *>(smem + OFF_SK + row * 256) + (c - 16);
-            else if (c < 48)
-                dst = reinterpret_cast<uint4 *>(smem + OFF_SV + row * 256) + (c - 32);
+            if (c < QV)
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SQ + row * 2 * D) + c;
+            else if (c < 2 * QV)
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SK + row * 2 * D) + (c - QV);
+            else if (c < 3 * QV)
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SV + row * 2 * D) + (c - 2 * QV);
             else
-                dst = reinterpret_cast<uint4 *>(smem + OFF_SG + row * 512) + (c - 48);
+                dst = reinterpret_cast<uint4 *>(smem + OFF_SG + row * 4 * D) + (c - 3 * QV);
             *dst = make_uint4(0u, 0u, 0u, 0u);
         }
         if (builders_only)
@@ -250,17 +266,20 @@ __device__ __forceinline__ void zero_tail(uint8_t *smem, int L, bool builders_on
 
 
 // ---- fast operands of a staged long segment into set `par` (builder warps).  Thread
-// (dp, qt) owns key dims 2dp, 2dp+1 for tokens [16 qt, 16 qt + 16): it sums their
-// log2-gates, then runs the cumulative sum again from the earlier quarters' totals (shared
-// memory; 2^{Lam_last} into gam slot `gslot`) while it writes Q~ and K~ (token-major, the
-// d-contractions' operands) and K~^T (rows of [A ; K~^T]), fp16, with 4- and 16-byte
-// stores.  Then thread (e, half) packs V^T into TMEM.  Per warp: max |q|, |k|, |v| and
-// whether every operand fits fp16 (for the guard).  The diagonal A_ii = q_i . k_i (no decay
-// between a token and itself) is summed in float32 from the bf16 inputs, each warp's 64 key
-// dims by a butterfly, into the set's diagonal partials: fp16 Q~ and K~ would round the
-// terms of that dot product to 11 bits, which a token whose own q . k cancels cannot afford.
+// (dp, qt) owns key dims 2dp, 2dp+1 for the TPG tokens of group qt (16 tokens x 4 groups at
+// D = 128, 8 x 8 at D = 64): it sums their log2-gates, then runs the cumulative sum again
+// from the earlier groups' totals (shared memory; 2^{Lam_last} into gam slot `gslot`) while
+// it writes Q~ and K~ (token-major, the d-contractions' operands) and K~^T (rows of
+// [A ; K~^T]), fp16, with 4- and 16-byte stores.  Then thread (e, half) packs V^T into TMEM
+// (zeros in the lanes e >= D).  Per warp: max |q|, |k|, |v| and whether every operand fits
+// fp16 (for the guard).  The diagonal A_ii = q_i . k_i (no decay between a token and itself)
+// is summed in float32 from the bf16 inputs, each warp's 64 key dims by a butterfly, into
+// the set's diagonal partials: fp16 Q~ and K~ would round the terms of that dot product to
+// 11 bits, which a token whose own q . k cancels cannot afford.
+template <int D>
 __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, int par, int gslot)
 {
+    using G = Geo<D>;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool worker = warp < 8;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
@@ -277,15 +296,15 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
 
     if (!worker)
         return;
-    zero_tail(smem, L, true);
-    const int dp = tid & 63, qt = (tid >> 6) & 3;
+    zero_tail<D>(smem, L, true);
+    const int dp = tid % G::DP, qt = tid / G::DP;
     float amax = -INFINITY;
     {
-        // quarter totals
+        // group totals
         float r0 = 0.f, r1 = 0.f;
 #pragma unroll
-        for (int x = 0; x < 16; ++x) {
-            const float2 a = *reinterpret_cast<const float2 *>(sG + (16 * qt + x) * D + 2 * dp);
+        for (int x = 0; x < G::TPG; ++x) {
+            const float2 a = *reinterpret_cast<const float2 *>(sG + (G::TPG * qt + x) * D + 2 * dp);
             amax = fmaxf(amax, fmaxf(a.x, a.y));
             r0 = fmaf(a.x, kLog2e, r0);
             r1 = fmaf(a.y, kLog2e, r1);
@@ -293,13 +312,13 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
         *reinterpret_cast<float2 *>(sTot + qt * D + 2 * dp) = make_float2(r0, r1);
     }
     bar_builders();
-    // the running sums start from the earlier quarters' totals
+    // the running sums start from the earlier groups' totals
     float run0 = 0.f, run1 = 0.f;
     bool lam_ok;
     {
         float t0 = 0.f, t1 = 0.f;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < G::NQ; ++u) {
             const float2 t = *reinterpret_cast<const float2 *>(sTot + u * D + 2 * dp);
             if (u < qt) {
                 run0 += t.x;
@@ -316,19 +335,19 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
     const int rowK = par ? 0 : 64;
     __nv_bfloat162 bq = __float2bfloat162_rn(0.f), bk = bq;   // max |q|, |k|
     __half2 hq = __float2half2_rn(0.f), hk = hq;                 // max |Q~|, |K~| (fp16)
-    // two groups of 8 tokens; within a group, token pairs: Q~ and K~ as fp16 pairs of key
-    // dims, K~^T rows 2dp and 2dp+1 as fp16 pairs of tokens (byte permutes of the K~ pairs)
-    float *sDg = reinterpret_cast<float *>(smem + OFF_DG) + par * 128 + (warp & 1) * 64;
+    // runs of 8 tokens; within a run, token pairs: Q~ and K~ as fp16 pairs of key dims,
+    // K~^T rows 2dp and 2dp+1 as fp16 pairs of tokens (byte permutes of the K~ pairs)
+    float *sDg = reinterpret_cast<float *>(smem + OFF_DG) + par * 128 + (dp >> 5) * 64;
 #pragma unroll 1
-    for (int grp = 0; grp < 2; ++grp) {
+    for (int grp = 0; grp < G::TPG / 8; ++grp) {
         uint32_t kt0[4], kt1[4];
-        float pd[8];   // q . k over this thread's two key dims, tokens 8 grp + 0..7 of its quarter
+        float pd[8];   // q . k over this thread's two key dims, tokens 8 grp + 0..7 of its group
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
             uint32_t kp[2];
 #pragma unroll
             for (int t = 0; t < 2; ++t) {
-                const int i = 16 * qt + 8 * grp + 2 * u + t;
+                const int i = G::TPG * qt + 8 * grp + 2 * u + t;
                 const float2 a = *reinterpret_cast<const float2 *>(sG + i * D + 2 * dp);
                 run0 = fmaf(a.x, kLog2e, run0);
                 run1 = fmaf(a.y, kLog2e, run1);
@@ -349,15 +368,15 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
             kt0[u] = __byte_perm(kp[0], kp[1], 0x5410);   // key dim 2dp: tokens (2u, 2u+1)
             kt1[u] = __byte_perm(kp[0], kp[1], 0x7632);   // key dim 2dp+1
         }
-        const int j0 = 16 * qt + 8 * grp;
+        const int j0 = G::TPG * qt + 8 * grp;
         {
             const float dsum = warp_sum8(pd, lane);
             if ((lane & 3) == 0)
                 sDg[j0 + ((lane >> 2) & 7)] = dsum;
         }
-        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowK + 2 * dp, j0)) =
+        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(G::ROWS, rowK + 2 * dp, j0)) =
             make_uint4(kt0[0], kt0[1], kt0[2], kt0[3]);
-        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowK + 2 * dp + 1, j0)) =
+        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(G::ROWS, rowK + 2 * dp + 1, j0)) =
             make_uint4(kt1[0], kt1[1], kt1[2], kt1[3]);
     }
     // V^T: thread (e, half) packs tokens [32 half, 32 half + 32) of value dim e
@@ -367,7 +386,9 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
 #pragma unroll
         for (int m = 0; m < 16; ++m) {
             const int i = 32 * th + 2 * m;
-            const uint32_t w = (uint32_t)sV[i * D + e_own] | ((uint32_t)sV[(i + 1) * D + e_own] << 16);
+            uint32_t w = 0;
+            if (e_own < D)
+                w = (uint32_t)sV[i * D + e_own] | ((uint32_t)sV[(i + 1) * D + e_own] << 16);
             bv = bmax_abs(bv, w);
             vpk[m] = pack_h2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
         }
@@ -376,7 +397,7 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
     float mq = warp_max(bmax_of(bq));
     float mk = warp_max(bmax_of(bk));
     float mv = warp_max(bmax_of(bv));
-    // non-increasing Lam (|Q~| <= |q|, |A| <= 128 max|q| max|k|), a total decay of at most
+    // non-increasing Lam (|Q~| <= |q|, |A| <= D max|q| max|k|), a total decay of at most
     // 2^-10 (Q~ of the segment's last tokens keeps its precision) and every fp16 operand below
     // 2^15; NaN fails
     bool ok = amax <= 0.f && lam_ok && hmax_of(hq) < kF16Lim && hmax_of(hk) < kF16Lim &&
@@ -394,8 +415,10 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
 
 // ---- state pass (state warps): decay by gam slot gpar (gpar < 0: none), checkpoint slot,
 // fp16 copy of S^T for the next S^T Q~^T, and the largest |S|
+template <int D>
 __device__ __forceinline__ void state_pass(uint8_t *smem, uint32_t tmem, int gpar, float *slot, bool copy)
 {
+    constexpr int CW = Geo<D>::CW;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const bool worker = warp >= 8;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;   // this warp's TMEM lane quarter
@@ -406,51 +429,54 @@ __device__ __forceinline__ void state_pass(uint8_t *smem, uint32_t tmem, int gpa
 
     if (!worker)
         return;
-    const int db = colhalf * 64;
-    float r[64];
-    tmem_ld32(tmem + lrow + TM_S + db, *reinterpret_cast<float(*)[32]>(&r[0]));
-    tmem_ld32(tmem + lrow + TM_S + db + 32, *reinterpret_cast<float(*)[32]>(&r[32]));
-    tmem_wait_ld();
-    if (gpar >= 0) {
-        const float *gam = sGam + gpar * D + db;
+    float m = 0.f;
+    if (e_own < D) {
+        const int db = colhalf * CW;
+        float r[CW];
 #pragma unroll
-        for (int c = 0; c < 16; ++c) {
-            const float4 g4 = *reinterpret_cast<const float4 *>(gam + 4 * c);
-            r[4 * c] *= g4.x;
-            r[4 * c + 1] *= g4.y;
-            r[4 * c + 2] *= g4.z;
-            r[4 * c + 3] *= g4.w;
-        }
-        tmem_st32(tmem + lrow + TM_S + db, *reinterpret_cast<float(*)[32]>(&r[0]));
-        tmem_st32(tmem + lrow + TM_S + db + 32, *reinterpret_cast<float(*)[32]>(&r[32]));
-    }
-    if (slot != nullptr) {
+        for (int c0 = 0; c0 < CW; c0 += 32)
+            tmem_ld32(tmem + lrow + TM_S + db + c0, *reinterpret_cast<float(*)[32]>(&r[c0]));
+        tmem_wait_ld();
+        if (gpar >= 0) {
+            const float *gam = sGam + gpar * D + db;
 #pragma unroll
-        for (int x = 0; x < 64; ++x)
-            slot[(int64_t)(db + x) * D + e_own] = r[x];
-    }
-    float m;
-    if (copy) {
-        // the fp16 copy, two key dims per column; its largest magnitude (inf past fp16)
-        __half2 hm = __float2half2_rn(0.f);
-#pragma unroll
-        for (int hh = 0; hh < 2; ++hh) {
-            uint32_t u[16];
-#pragma unroll
-            for (int c = 0; c < 16; ++c) {
-                u[c] = pack_h2(r[32 * hh + 2 * c], r[32 * hh + 2 * c + 1]);
-                hm = hmax_abs(hm, u[c]);
+            for (int c = 0; c < CW / 4; ++c) {
+                const float4 g4 = *reinterpret_cast<const float4 *>(gam + 4 * c);
+                r[4 * c] *= g4.x;
+                r[4 * c + 1] *= g4.y;
+                r[4 * c + 2] *= g4.z;
+                r[4 * c + 3] *= g4.w;
             }
-            tmem_st16(tmem + lrow + TM_SH + db / 2 + 16 * hh, u);
-        }
-        m = hmax_of(hm);
-    } else {
-        m = 0.f;
 #pragma unroll
-        for (int x = 0; x < 64; ++x)
-            m = fmaxf(m, fabsf(r[x]));
+            for (int c0 = 0; c0 < CW; c0 += 32)
+                tmem_st32(tmem + lrow + TM_S + db + c0, *reinterpret_cast<float(*)[32]>(&r[c0]));
+        }
+        if (slot != nullptr) {
+#pragma unroll
+            for (int x = 0; x < CW; ++x)
+                slot[(int64_t)(db + x) * D + e_own] = r[x];
+        }
+        if (copy) {
+            // the fp16 copy, two key dims per column; its largest magnitude (inf past fp16)
+            __half2 hm = __float2half2_rn(0.f);
+#pragma unroll
+            for (int hh = 0; hh < CW / 32; ++hh) {
+                uint32_t u[16];
+#pragma unroll
+                for (int c = 0; c < 16; ++c) {
+                    u[c] = pack_h2(r[32 * hh + 2 * c], r[32 * hh + 2 * c + 1]);
+                    hm = hmax_abs(hm, u[c]);
+                }
+                tmem_st16(tmem + lrow + TM_SH + db / 2 + 16 * hh, u);
+            }
+            m = hmax_of(hm);
+        } else {
+#pragma unroll
+            for (int x = 0; x < CW; ++x)
+                m = fmaxf(m, fabsf(r[x]));
+        }
+        tmem_wait_st();
     }
-    tmem_wait_st();
     m = warp_max(m);
     if (lane == 0)
         sRed[(warp & 7) * 8 + 4] = m;
@@ -459,6 +485,7 @@ __device__ __forceinline__ void state_pass(uint8_t *smem, uint32_t tmem, int gpa
 
 // ---- the causally masked intra-chunk matrix A (D_A) -> rows rowA.. of set par's [A ; K~^T]
 // (state warps of TMEM lane quarters 0 and 1)
+template <int D>
 __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
 {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -469,12 +496,12 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
         return;
     const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
     const int jb = ((warp >> 2) & 1) * 32;      // this warp's 32 key columns
-    const int rowA = par ? 128 : 0;
+    const int rowA = par ? D : 0;
     float r[32];
     tmem_ld32(tmem + lrow + (par ? TM_A1 : TM_A0) + jb, r);
-    // the diagonal from the builders' float32 partials (the two key-dim halves)
+    // the diagonal from the builders' float32 partials (one per 64 key dims)
     const float *sDg = reinterpret_cast<const float *>(smem + OFF_DG) + par * 128;
-    const float dg = (i >= jb && i < jb + 32) ? sDg[i] + sDg[64 + i] : 0.f;
+    const float dg = (i >= jb && i < jb + 32) ? (D == 128 ? sDg[i] + sDg[64 + i] : sDg[i]) : 0.f;
     tmem_wait_ld();
     uint8_t *set = smem + par * SET_BYTES;
 #pragma unroll
@@ -487,7 +514,7 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
             const float x1 = j0 + 1 == i ? dg : (j0 + 1 <= i ? r[8 * c + 2 * u + 1] : 0.f);
             w[u] = pack_h2(x0, x1);
         }
-        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(192, rowA + i, jb + 8 * c)) =
+        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(Geo<D>::ROWS, rowA + i, jb + 8 * c)) =
             make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
@@ -496,6 +523,7 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
 // ---- output epilogue of a processed segment (state warps): D_O buffer `par` -> o (lane e,
 // 32 rows per warp).  With `spare_issuer`, the warp of the MMA-issuing thread (warp 8) is
 // left out while it issues, and warp 12 (the same TMEM lane quarter) writes both halves.
+template <int D>
 __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t tstride, int L, int par,
                                              bool spare_issuer)
 {
@@ -505,7 +533,7 @@ __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t t
     const int colhalf = (warp >> 2) & 1;
     const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
 
-    if (!worker || (spare_issuer && warp == 8))
+    if (!worker || (spare_issuer && warp == 8) || e_own >= D)
         return;
     const int h0 = (spare_issuer && warp == 12) ? 0 : colhalf;
     const int h1 = (spare_issuer && warp == 12) ? 2 : colhalf + 1;
@@ -513,7 +541,7 @@ __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t t
     for (int hh = h0; hh < h1; ++hh) {
         float r[32];
         const int ib = hh * 32;
-        tmem_ld32(tmem + lrow + (par ? TM_O1 : TM_O0) + ib, r);
+        tmem_ld32(tmem + lrow + (par ? Geo<D>::O1 : TM_O0) + ib, r);
         tmem_wait_ld();
         float *op = ob + (int64_t)ib * tstride + e_own;
         if (L == CH) {
@@ -533,8 +561,10 @@ __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t t
 // ---- the state between global memory ([d][e], row = key dim) and TMEM (S^T, lane e) ----
 
 // (state warps) load a state into TMEM and record its largest |S| (float32) for the guard
+template <int D>
 __device__ __forceinline__ void state_load(uint8_t *smem, uint32_t tmem, const float *src)
 {
+    constexpr int CW = Geo<D>::CW;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     if (warp < 8)
         return;
@@ -544,35 +574,39 @@ __device__ __forceinline__ void state_load(uint8_t *smem, uint32_t tmem, const f
     float *sRed = reinterpret_cast<float *>(smem + OFF_RED);
     float r[32];
     float m = 0.f;
+    if (e_own < D) {
 #pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 32) {
-        const int d0 = colhalf * 64 + c0;
+        for (int c0 = 0; c0 < CW; c0 += 32) {
+            const int d0 = colhalf * CW + c0;
 #pragma unroll
-        for (int x = 0; x < 32; ++x) {
-            r[x] = src[(int64_t)(d0 + x) * D + e_own];
-            m = fmaxf(m, fabsf(r[x]));
+            for (int x = 0; x < 32; ++x) {
+                r[x] = src[(int64_t)(d0 + x) * D + e_own];
+                m = fmaxf(m, fabsf(r[x]));
+            }
+            tmem_st32(tmem + lrow + TM_S + d0, r);
         }
-        tmem_st32(tmem + lrow + TM_S + d0, r);
+        tmem_wait_st();
     }
-    tmem_wait_st();
     m = warp_max(m);
     if (lane == 0)
         sRed[(warp & 7) * 8 + 4] = m;
 }
 
 // (state warps) store the state in TMEM to global memory
+template <int D>
 __device__ __forceinline__ void state_store(uint32_t tmem, float *dst)
 {
+    constexpr int CW = Geo<D>::CW;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (warp < 8)
+    const int e_own = (warp & 3) * 32 + lane;
+    if (warp < 8 || e_own >= D)
         return;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
     const int colhalf = (warp >> 2) & 1;
-    const int e_own = (warp & 3) * 32 + lane;
     float r[32];
 #pragma unroll
-    for (int c0 = 0; c0 < 64; c0 += 32) {
-        const int d0 = colhalf * 64 + c0;
+    for (int c0 = 0; c0 < CW; c0 += 32) {
+        const int d0 = colhalf * CW + c0;
         tmem_ld32(tmem + lrow + TM_S + d0, r);
         tmem_wait_ld();
 #pragma unroll
@@ -587,13 +621,14 @@ __device__ __forceinline__ void state_store(uint32_t tmem, float *dst)
 // token-major into X_LAM; gates below kGateFloor taken at the floor), Q~ = q 2^{Lam} (tf32,
 // X_QT), K^^T = k 2^{Lam_last - Lam} (tf32, rows 64.. of X_B2), V^T float32 into TMEM and
 // 2^{Lam_last} into gam slot gslot.  Ends with the operands visible to the tensor core.
+template <int D>
 __device__ __forceinline__ void exact_build(uint8_t *smem, uint32_t tmem, int L, int gslot)
 {
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool worker = warp >= 8;
+    const int d = (warp & 3) * 32 + lane;
+    const bool worker = warp >= 8 && d < D;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
     const int colhalf = (warp >> 2) & 1;
-    const int d = (warp & 3) * 32 + lane;
     const int th = colhalf;
     const uint16_t *sQ = reinterpret_cast<const uint16_t *>(smem + OFF_SQ);
     const uint16_t *sK = reinterpret_cast<const uint16_t *>(smem + OFF_SK);
@@ -603,7 +638,7 @@ __device__ __forceinline__ void exact_build(uint8_t *smem, uint32_t tmem, int L,
     float *sGam = reinterpret_cast<float *>(smem + OFF_GAM);
     float *sLam = reinterpret_cast<float *>(smem + X_LAM);
     float last = 0.f, tot0 = 0.f;
-    zero_tail(smem, L, false);
+    zero_tail<D>(smem, L, false);
     {
         float run = 0.f;
         if (worker) {
@@ -644,7 +679,7 @@ __device__ __forceinline__ void exact_build(uint8_t *smem, uint32_t tmem, int L,
                     wv[u] = rna_tf32(bf16f(sK[i * D + d]) * ex2(last - lam));
                     vtr[4 * g + u] = __float_as_uint(bf16f(sV[i * D + d]));
                 }
-                *reinterpret_cast<float4 *>(smem + X_B2 + t_off(192, 64 + d, 32 * th + 16 * hh + 4 * g)) = w;
+                *reinterpret_cast<float4 *>(smem + X_B2 + t_off(Geo<D>::ROWS, 64 + d, 32 * th + 16 * hh + 4 * g)) = w;
             }
             tmem_st16(tmem + lrow + TM_V + 32 * th + 16 * hh, vtr);
         }
@@ -656,16 +691,18 @@ __device__ __forceinline__ void exact_build(uint8_t *smem, uint32_t tmem, int L,
 // tf32): hi = S with its low 13 mantissa bits cleared (exact in tf32), lo = S - hi (exact in
 // fp32, at most 13 significant bits), so the product keeps the state to ~2^-20 instead of a
 // 2^-10 truncation
+template <int D>
 __device__ __forceinline__ void exact_split_state(uint32_t tmem)
 {
-    const int warp = threadIdx.x >> 5;
-    if (warp < 8)
+    constexpr int CW = Geo<D>::CW;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (warp < 8 || (warp & 3) * 32 + lane >= D)
         return;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
     const int colhalf = (warp >> 2) & 1;
 #pragma unroll 1
-    for (int c0 = 0; c0 < 64; c0 += 32) {
-        const int d0 = colhalf * 64 + c0;
+    for (int c0 = 0; c0 < CW; c0 += 32) {
+        const int d0 = colhalf * CW + c0;
         float r[32], lo[32];
         tmem_ld32(tmem + lrow + TM_S + d0, r);
         tmem_wait_ld();
@@ -675,19 +712,20 @@ __device__ __forceinline__ void exact_split_state(uint32_t tmem)
             lo[x] = r[x] - hi;
             r[x] = hi;
         }
-        tmem_st32(tmem + lrow + TM_SHI + d0, r);
+        tmem_st32(tmem + lrow + Geo<D>::SHI + d0, r);
         tmem_st32(tmem + lrow + (d0 < 64 ? TM_SLO0 + d0 : TM_SLO1 + (d0 - 64)), lo);
     }
     tmem_wait_st();
 }
 
 // (issuing thread) S^T Q~^T into D_O (TM_O0): the hi part, then the lo part
+template <int D>
 __device__ __forceinline__ void exact_issue_sq(uint32_t tmem, uint32_t sb)
 {
 #pragma unroll 1
     for (int kk = 0; kk < D / 8; ++kk) {
         const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
-        mma_tf32_ts(tmem + TM_O0, tmem + TM_SHI + kk * 8, sdesc_sw128(sb + X_QT + koff, 16, 1024),
+        mma_tf32_ts(tmem + TM_O0, tmem + Geo<D>::SHI + kk * 8, sdesc_sw128(sb + X_QT + koff, 16, 1024),
                     IDT_N64, kk > 0);
     }
 #pragma unroll 1
@@ -700,6 +738,7 @@ __device__ __forceinline__ void exact_issue_sq(uint32_t tmem, uint32_t sb)
 
 // (every thread) A_ij = sum_d q_id k_jd 2^{Lam_id - Lam_jd}, j <= i < L, elementwise, rounded
 // to tf32 into rows 0..63 of X_B2
+template <int D>
 __device__ __forceinline__ void exact_scores(uint8_t *smem, int L)
 {
     const int tid = threadIdx.x;
@@ -714,35 +753,38 @@ __device__ __forceinline__ void exact_scores(uint8_t *smem, int L)
                 acc = fmaf(bf16f(sQ[i * D + dd]) * bf16f(sK[j * D + dd]),
                            ex2(lg[i * D + dd] - lg[j * D + dd]), acc);
         }
-        *reinterpret_cast<float *>(smem + X_B2 + t_off(192, i, j)) = rna_tf32(acc);
+        *reinterpret_cast<float *>(smem + X_B2 + t_off(Geo<D>::ROWS, i, j)) = rna_tf32(acc);
     }
 }
 
 // (issuing thread) D_O += V^T A^T
+template <int D>
 __device__ __forceinline__ void exact_issue_av(uint32_t tmem, uint32_t sb)
 {
 #pragma unroll
     for (int kk = 0; kk < CH / 8; ++kk) {
-        const uint32_t koff = (kk >> 2) * (192 * 128) + (kk & 3) * 32;
+        const uint32_t koff = (kk >> 2) * (Geo<D>::ROWS * 128) + (kk & 3) * 32;
         mma_tf32_ts(tmem + TM_O0, tmem + TM_V + kk * 8, sdesc_sw128(sb + X_B2 + koff, 16, 1024),
                     IDT_N64, 1);
     }
 }
 
 // (issuing thread) S^T += V^T K^ (the decay diag(2^{Lam_last}) S applied before)
+template <int D>
 __device__ __forceinline__ void exact_issue_state(uint32_t tmem, uint32_t sb)
 {
 #pragma unroll
     for (int kk = 0; kk < CH / 8; ++kk) {
-        const uint32_t koff = (kk >> 2) * (192 * 128) + (kk & 3) * 32 + 64 * 128;
+        const uint32_t koff = (kk >> 2) * (Geo<D>::ROWS * 128) + (kk & 3) * 32 + 64 * 128;
         mma_tf32_ts(tmem + TM_S, tmem + TM_V + kk * 8, sdesc_sw128(sb + X_B2 + koff, 16, 1024),
-                    IDT_N128, 1);
+                    Geo<D>::IDT_ST, 1);
     }
 }
 
 // ---- fast path MMA groups (issuing thread) ----
 
 // D_A = Q~ K~^T of operand set `par` into its own buffer
+template <int D>
 __device__ __forceinline__ void fast_issue_scores(uint32_t tmem, uint32_t sb, int par)
 {
     const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
@@ -754,20 +796,22 @@ __device__ __forceinline__ void fast_issue_scores(uint32_t tmem, uint32_t sb, in
     }
 }
 
-// D_O = S^T Q~^T (A operand: the fp16 copy of S^T; the N = 192 product accumulates onto it)
+// D_O = S^T Q~^T (A operand: the fp16 copy of S^T; the update product accumulates onto it)
+template <int D>
 __device__ __forceinline__ void fast_issue_sq(uint32_t tmem, uint32_t sb, int par)
 {
     const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
 #pragma unroll 1
     for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t koff = (kk >> 2) * 8192 + (kk & 3) * 32;
-        mma_f16_ts(tmem + (par ? TM_O1 : TM_O0), tmem + TM_SH + kk * 8,
+        mma_f16_ts(tmem + (par ? Geo<D>::O1 : TM_O0), tmem + TM_SH + kk * 8,
                    sdesc_sw128(setb + S_QH + koff, 16, 1024), IDF_N64, kk > 0);
     }
 }
 
-// [D_O | S^T] += V^T [A ; K~^T]^T as one N = 192 product (even sets order the operand's rows
-// [A ; K~^T] with D_O0 on the left of S^T, odd sets [K~^T ; A] with D_O1 on the right)
+// [D_O | S^T] += V^T [A ; K~^T]^T as one N = 64 + D product (even sets order the operand's
+// rows [A ; K~^T] with D_O0 on the left of S^T, odd sets [K~^T ; A] with D_O1 on the right)
+template <int D>
 __device__ __forceinline__ void fast_issue_update(uint32_t tmem, uint32_t sb, int par)
 {
     const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
@@ -775,7 +819,7 @@ __device__ __forceinline__ void fast_issue_update(uint32_t tmem, uint32_t sb, in
 #pragma unroll 1
     for (int kk = 0; kk < CH / 16; ++kk)
         mma_f16_ts(tmem + (par ? TM_S : TM_O0), vt + kk * 8,
-                   sdesc_sw128(setb + S_B2H + kk * 32, 16, 1024), IDF_N192, 1);
+                   sdesc_sw128(setb + S_B2H + kk * 32, 16, 1024), Geo<D>::IDF_UPD, 1);
 }
 
 // ---- short segments (<= kShort tokens): the per-token recurrence with the recurrent kernel's
@@ -783,13 +827,15 @@ __device__ __forceinline__ void fast_issue_update(uint32_t tmem, uint32_t sb, in
 // right).  The state part (every thread; gates exponentiated in place, then the state warps
 // update S in TMEM, write the slot and the largest |S|, and leave each token's group partials
 // in the operand sets) ...
+template <int D>
 __device__ __forceinline__ void short_state(uint8_t *smem, uint32_t tmem, int L, float *slot)
 {
+    constexpr int CW = Geo<D>::CW, NG = Geo<D>::NG;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const bool worker = warp >= 8;
+    const int e_own = (warp & 3) * 32 + lane;
+    const bool worker = warp >= 8 && e_own < D;
     const uint32_t lrow = (uint32_t)((warp & 3) * 32) << 16;
     const int colhalf = (warp >> 2) & 1;
-    const int e_own = (warp & 3) * 32 + lane;
     const uint16_t *sQ = reinterpret_cast<const uint16_t *>(smem + OFF_SQ);
     const uint16_t *sK = reinterpret_cast<const uint16_t *>(smem + OFF_SK);
     const uint16_t *sV = reinterpret_cast<const uint16_t *>(smem + OFF_SV);
@@ -798,39 +844,43 @@ __device__ __forceinline__ void short_state(uint8_t *smem, uint32_t tmem, int L,
     for (int idx = tid; idx < L * D; idx += NT)
         sG[idx] = expf(sG[idx]);
     __syncthreads();
-    float *part = reinterpret_cast<float *>(smem);   // [kShort][8 groups][128] in the operand sets
-    if (worker) {
-        float S[64];
-        tmem_ld32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
-        tmem_ld32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
-        tmem_wait_ld();
-        for (int i = 0; i < L; ++i) {
-            const float ve = bf16f(sV[i * D + e_own]);
-#pragma unroll
-            for (int m = 0; m < 4; ++m) {
-                float acc = 0.f;
-#pragma unroll
-                for (int r = 16 * m; r < 16 * m + 16; ++r) {
-                    const int dd = colhalf * 64 + r;
-                    S[r] = fmaf(sG[i * D + dd], S[r], bf16f(sK[i * D + dd]) * ve);
-                    acc = fmaf(bf16f(sQ[i * D + dd]), S[r], acc);
-                }
-                part[(i * 8 + colhalf * 4 + m) * D + e_own] = acc;
-            }
-        }
-        tmem_st32(tmem + lrow + TM_S + colhalf * 64, *reinterpret_cast<float(*)[32]>(&S[0]));
-        tmem_st32(tmem + lrow + TM_S + colhalf * 64 + 32, *reinterpret_cast<float(*)[32]>(&S[32]));
+    float *part = reinterpret_cast<float *>(smem);   // [kShort][D/16 groups][D] in the operand sets
+    if (warp >= 8) {
         float m = 0.f;
+        if (worker) {
+            float S[CW];
 #pragma unroll
-        for (int r = 0; r < 64; ++r) {
-            m = fmaxf(m, fabsf(S[r]));
-            if (slot != nullptr)
-                slot[(int64_t)(colhalf * 64 + r) * D + e_own] = S[r];
+            for (int c0 = 0; c0 < CW; c0 += 32)
+                tmem_ld32(tmem + lrow + TM_S + colhalf * CW + c0, *reinterpret_cast<float(*)[32]>(&S[c0]));
+            tmem_wait_ld();
+            for (int i = 0; i < L; ++i) {
+                const float ve = bf16f(sV[i * D + e_own]);
+#pragma unroll
+                for (int mm = 0; mm < CW / 16; ++mm) {
+                    float acc = 0.f;
+#pragma unroll
+                    for (int r = 16 * mm; r < 16 * mm + 16; ++r) {
+                        const int dd = colhalf * CW + r;
+                        S[r] = fmaf(sG[i * D + dd], S[r], bf16f(sK[i * D + dd]) * ve);
+                        acc = fmaf(bf16f(sQ[i * D + dd]), S[r], acc);
+                    }
+                    part[(i * NG + colhalf * (NG / 2) + mm) * D + e_own] = acc;
+                }
+            }
+#pragma unroll
+            for (int c0 = 0; c0 < CW; c0 += 32)
+                tmem_st32(tmem + lrow + TM_S + colhalf * CW + c0, *reinterpret_cast<float(*)[32]>(&S[c0]));
+#pragma unroll
+            for (int r = 0; r < CW; ++r) {
+                m = fmaxf(m, fabsf(S[r]));
+                if (slot != nullptr)
+                    slot[(int64_t)(colhalf * CW + r) * D + e_own] = S[r];
+            }
+            tmem_wait_st();
         }
         m = warp_max(m);
         if (lane == 0)
             sRed[(warp & 7) * 8 + 4] = m;
-        tmem_wait_st();
     }
     fence_proxy_async_smem();
     __syncthreads();
@@ -838,15 +888,17 @@ __device__ __forceinline__ void short_state(uint8_t *smem, uint32_t tmem, int L,
 
 // ... and the outputs (every thread): each token's output is the left-to-right sum of its
 // eight group partials
+template <int D>
 __device__ __forceinline__ void short_outputs(const uint8_t *smem, int L, float *ob, int64_t tstride)
 {
+    constexpr int NG = Geo<D>::NG;
     const float *part = reinterpret_cast<const float *>(smem);
     for (int idx = threadIdx.x; idx < L * D; idx += NT) {
-        const int i = idx >> 7, e = idx & (D - 1);
-        float sum = part[(i * 8) * D + e];
+        const int i = idx / D, e = idx % D;
+        float sum = part[(i * NG) * D + e];
 #pragma unroll
-        for (int g = 1; g < 8; ++g)
-            sum += part[(i * 8 + g) * D + e];
+        for (int g = 1; g < NG; ++g)
+            sum += part[(i * NG + g) * D + e];
         ob[(int64_t)i * tstride + e] = sum;
     }
 }
@@ -869,8 +921,9 @@ inline PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
+template <int D>
 inline bool encode_rows(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t inner,
-                 uint64_t rows, uint32_t elem)
+                        uint64_t rows, uint32_t elem)
 {
     auto fn = encode_fn();
     if (fn == nullptr)

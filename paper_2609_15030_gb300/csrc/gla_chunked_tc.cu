@@ -55,6 +55,7 @@ namespace {
 using namespace ptx;
 using namespace gck;
 
+template <int D>
 __global__ void __launch_bounds__(NT, 1)
 gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant__ TmaMaps maps)
 {
@@ -141,7 +142,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     auto issue_tma = [&](int64_t tok_local) {
         const int32_t y = (int32_t)((int64_t)p.row0[b] + tok_local);
         const int32_t x = h * D;
-        mbar_arrive_expect_tx(bar_tma, STAGE_BYTES);
+        mbar_arrive_expect_tx(bar_tma, Geo<D>::STAGE);
         tma_load_2d(sb + OFF_SQ, &maps.q, x, y, bar_tma);
         tma_load_2d(sb + OFF_SK, &maps.k, x, y, bar_tma);
         tma_load_2d(sb + OFF_SV, &maps.v, x, y, bar_tma);
@@ -227,7 +228,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // largest magnitude.  The builders meanwhile stage and build the first segment.
     float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
     if (worker) {
-        state_load(smem, tmem, st_g);
+        state_load<D>(smem, tmem, st_g);
         tc_fence_before();
         bar_staters();
         tc_fence_after();
@@ -237,10 +238,10 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // pending): the per-token recurrence with the recurrent kernel's exact operation order
     // (fma chains over groups of 16 key rows, group partials summed left to right)
     auto short_segment = [&](int64_t tok_s, int L, int64_t seg_end) {
-        short_state(smem, tmem, L, ckpt_slot(seg_end));
+        short_state<D>(smem, tmem, L, ckpt_slot(seg_end));
         if (tid == kLoader && seg_end < end)
             issue_tma(tok_s + L);
-        short_outputs(smem, L, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride);
+        short_outputs<D>(smem, L, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride);
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -264,44 +265,44 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         mk_new = mk;
         mv_new = mv;
         state_ok = s_mag < kF16Lim;
-        return ok && 128.0f * mq * mk < kF16Lim;
+        return ok && (float)D * mq * mk < kF16Lim;
     };
 
     // ---- one exact segment, from staged inputs, no decay pending and no MMA in flight;
     // leaves the final state in TMEM, writes its outputs and checkpoint
     auto exact_segment = [&](int64_t tok_s, int L, int par, int gslot, int64_t seg_end) -> bool {
-        exact_build(smem, tmem, L, gslot);
-        exact_split_state(tmem);
+        exact_build<D>(smem, tmem, L, gslot);
+        exact_split_state<D>(tmem);
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
         if (tid == kIssuer) {
             tc_fence_after();
-            exact_issue_sq(tmem, sb);
+            exact_issue_sq<D>(tmem, sb);
         }
-        exact_scores(smem, L);
+        exact_scores<D>(smem, L);
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
         if (tid == kIssuer) {
             tc_fence_after();
-            exact_issue_av(tmem, sb);
+            exact_issue_av<D>(tmem, sb);
             tc_commit(bar_o);
         }
         if (!wait_all(kIssuer, bar_o, ph_o))
             return false;
-        state_pass(smem, tmem, gslot, nullptr, false);          // S <- diag(2^{Lam_last}) S
+        state_pass<D>(smem, tmem, gslot, nullptr, false);          // S <- diag(2^{Lam_last}) S
         tc_fence_before();
         __syncthreads();
         if (tid == kIssuer) {
             tc_fence_after();
-            exact_issue_state(tmem, sb);
+            exact_issue_state<D>(tmem, sb);
             tc_commit(bar_s);
         }
         if (!wait_all(kIssuer, bar_s, ph_s))
             return false;
-        state_pass(smem, tmem, -1, ckpt_slot(seg_end), false);   // checkpoint and |S| of the final state
-        out_epilogue(tmem, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride, L, par, false);
+        state_pass<D>(smem, tmem, -1, ckpt_slot(seg_end), false);   // checkpoint and |S| of the final state
+        out_epilogue<D>(tmem, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride, L, par, false);
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -337,7 +338,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 for (int j = 1; j <= kPrefetch; ++j)
                     prefetch(rtok + L + (int64_t)CH * (j - 1));
             }
-            build_fast(smem, tmem, L, par, kseq & 3);
+            build_fast<D>(smem, tmem, L, par, kseq & 3);
             fence_proxy_async_smem();
             tc_fence_before();
             if (!sync_group(1))
@@ -352,7 +353,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 // D_A = Q~ K~^T of this segment, into its own buffer (the state warps wait on
                 // bar_a / bar_a1 by parity before they read it)
                 tc_fence_after();
-                fast_issue_scores(tmem, sb, par);
+                fast_issue_scores<D>(tmem, sb, par);
                 tc_commit(par ? bar_a1 : bar_a);
             }
             if (!wait_group(1, kLoader, bar_go, ph_go))
@@ -397,28 +398,28 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             // the products of the previous segment are complete: its operand set is free
             if (tid == kIssuer)
                 mbar_arrive(bar_go);
-            state_pass(smem, tmem, pend ? pend_g : -1, pend ? ckpt_slot(pend_end) : nullptr, true);
+            state_pass<D>(smem, tmem, pend ? pend_g : -1, pend ? ckpt_slot(pend_end) : nullptr, true);
             tc_fence_before();
             if (!sync_group(2))
                 return;
             if (tid == kIssuer) {
                 // D_O = S^T Q~^T (the N = 192 product below accumulates onto it in order)
                 tc_fence_after();
-                fast_issue_sq(tmem, sb, par);
+                fast_issue_sq<D>(tmem, sb, par);
             }
             if (pend)
-                out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par, true);
+                out_epilogue<D>(tmem, outp(pend_tok), tstride, pend_L, pend_par, true);
             // D_A of this segment (issued by the builders' loader)
             if (!(par ? wait_group(2, kIssuer, bar_a1, ph_a1) : wait_group(2, kIssuer, bar_a, ph_a0)))
                 return;
-            a_build(smem, tmem, par);
+            a_build<D>(smem, tmem, par);
             fence_proxy_async_smem();
             tc_fence_before();
             if (!sync_group(2))
                 return;
             if (tid == kIssuer) {
                 tc_fence_after();
-                fast_issue_update(tmem, sb, par);
+                fast_issue_update<D>(tmem, sb, par);
                 tc_commit(bar_o);
             }
             pend = true;
@@ -453,8 +454,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (pend) {
             if (!wait_group(2, kIssuer, bar_o, ph_o))
                 return;
-            state_pass(smem, tmem, pend_g, ckpt_slot(pend_end), false);
-            out_epilogue(tmem, outp(pend_tok), tstride, pend_L, pend_par, false);
+            state_pass<D>(smem, tmem, pend_g, ckpt_slot(pend_end), false);
+            out_epilogue<D>(tmem, outp(pend_tok), tstride, pend_L, pend_par, false);
             tc_fence_before();
             if (!sync_group(2))
                 return;
@@ -524,7 +525,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     }
 
     if (!aborted) {
-        state_store(tmem, st_g);   // final state back to global memory, row = key dim
+        state_store<D>(tmem, st_g);   // final state back to global memory, row = key dim
     } else {
         // let this CTA's own copies and MMAs drain (bounded) before its memory goes away
         if (tid == kLoader) {
@@ -552,13 +553,14 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
 
 bool gla_chunked_tc_supported(int d)
 {
-    return d == D;
+    return d == 64 || d == 128;
 }
 
-cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s)
+namespace {
+
+template <int D>
+cudaError_t launch_tc(const GlaParams &p, cudaStream_t s)
 {
-    if (!gla_chunked_tc_supported(d))
-        return cudaErrorNotSupported;
     TmaMaps maps;
     const uint64_t inner = (uint64_t)p.n_heads * D;
     // rows up to the last token any problem has: copies never read beyond the tokens the
@@ -571,17 +573,28 @@ cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s)
     }
     if (rows == 0)
         return cudaSuccess;
-    if (!encode_rows(&maps.q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.q, inner, rows, 2) ||
-        !encode_rows(&maps.k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.k, inner, rows, 2) ||
-        !encode_rows(&maps.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.v, inner, rows, 2) ||
-        !encode_rows(&maps.g, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, p.log_g, inner, rows, 4))
+    if (!encode_rows<D>(&maps.q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.q, inner, rows, 2) ||
+        !encode_rows<D>(&maps.k, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.k, inner, rows, 2) ||
+        !encode_rows<D>(&maps.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.v, inner, rows, 2) ||
+        !encode_rows<D>(&maps.g, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, p.log_g, inner, rows, 4))
         return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(gla_chunked_tc_kernel,
+    cudaError_t e = cudaFuncSetAttribute(gla_chunked_tc_kernel<D>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
     if (e != cudaSuccess)
         return e;
     const unsigned grid = (unsigned)p.batch * (unsigned)p.n_heads;
-    return launch_pdl(gla_chunked_tc_kernel, dim3(grid), dim3(NT), SMEM_BYTES, s, p, maps);
+    return launch_pdl(gla_chunked_tc_kernel<D>, dim3(grid), dim3(NT), SMEM_BYTES, s, p, maps);
+}
+
+}  // namespace
+
+cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s)
+{
+    if (d == 128)
+        return launch_tc<128>(p, s);
+    if (d == 64)
+        return launch_tc<64>(p, s);
+    return cudaErrorNotSupported;
 }
 
 }  // namespace hs

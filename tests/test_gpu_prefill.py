@@ -22,9 +22,8 @@ KERNELS = [pytest.param(hs.HS_LINATTN_RECURRENT, id="recurrent"),
 
 
 def _needs(kernel, d):
-    """The tensor-core kernel implements d = 128 only (HS_ERR_UNSUPPORTED otherwise)."""
-    if kernel == hs.HS_LINATTN_CHUNKED_TC and d != 128:
-        pytest.skip("chunked tensor-core kernel: d = 128 only")
+    """Every kernel implements both head widths (d = 64 and 128)."""
+    assert d in (64, 128)
 
 
 def _check(o, S, cks, ro, rS, rcks, pos0, n_tokens, what=""):
@@ -66,6 +65,18 @@ def test_tiny_hybrid_config(kernel):
     o_f, S_f, ck_f = _resume_equals_recompute(inp, N, c, C, dev, kernel)
     ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], C_=C)
     _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], "tiny")
+
+
+def test_head_width_64_fast_path_resumes_bitwise():
+    """d = 64 on the tensor cores (M = 128 products with half the TMEM lanes unused): gates
+    U(-0.1, 0) keep every segment on the fp16 path; resuming from the checkpoint at 512
+    reproduces the recomputation bit for bit and both follow the oracle."""
+    dev = device()
+    N, C, nH, d = 1000, 128, 8, 64
+    inp = gen_linear(17, 0, 1, N, nH, d, d)
+    o_f, S_f, ck_f = _resume_equals_recompute(inp, N, 512, C, dev, hs.HS_LINATTN_CHUNKED_TC)
+    ro, rS, rck = oracle.gla(inp.q, inp.k, inp.v, inp.a, [0], [N], C_=C, threads=16)
+    _check(o_f, S_f, ck_f, ro, rS, rck, [0], [N], "d64 fast")
 
 
 @pytest.mark.parametrize("kernel", KERNELS)
@@ -313,10 +324,10 @@ def test_random_configurations(case):
     """Seeded random calls: batch 1-3, 1-3 heads, resume points anywhere in [0, 320), tails
     of 0-399 tokens, checkpoint interval 0/64/128/192, from a random state, with growing
     gates (the exact path) on up to two random token ranges; the tensor-core kernel and
-    AUTO against the oracle."""
+    AUTO against the oracle.  Odd cases use the head width 64."""
     dev = device()
     rng = np.random.default_rng(1000 + case)
-    B, nH, d = int(rng.integers(1, 4)), int(rng.integers(1, 4)), 128
+    B, nH, d = int(rng.integers(1, 4)), int(rng.integers(1, 4)), (128 if case % 2 == 0 else 64)
     C = int(rng.choice([0, 64, 128, 192]))
     pos0 = [int(x) for x in rng.integers(0, 320, B)]
     n_tok = [int(x) for x in rng.integers(0, 400, B)]
@@ -468,12 +479,13 @@ def test_long_context_full_size_sampled_heads(kernel, L):
         assert maxnorm_err(got_ck, rck[0][:, 0], axes=(1, 2)) <= TOL
 
 
-def test_short_segments_match_across_kernels():
+@pytest.mark.parametrize("d", [64, 128])
+def test_short_segments_match_across_kernels(d):
     """Calls whose tails are at most HS_SHORT_SEGMENT tokens: the tensor-core
     kernel's token-by-token path and the recurrent kernel agree bit for bit, so
     AUTO may send decode steps to either without changing results."""
     dev = device()
-    B, nH, d, T = 6, 4, 128, 8
+    B, nH, T = 6, 4, 8
     pos0 = [0, 5, 63, 64, 1000, 4095]
     n_tok = [8, 1, 2, 7, 3, 8]                       # some straddle a chunk boundary
     inp = gen_linear(13, 0, B, T, nH, d, d)
@@ -500,9 +512,8 @@ def test_single_token_steps_match_across_kernels(d):
     pos0 = [0, 61, 126, 4093, 700]      # problems 1-3 cross a 64-token boundary in these steps
     inp = gen_linear(21, d, B, steps, nH, d, d)
     S0 = gen_state(21, d, B, nH, d, d)
-    kernels = [hs.HS_LINATTN_SINGLE_TOKEN, hs.HS_LINATTN_RECURRENT, hs.HS_LINATTN_AUTO]
-    if d == 128:
-        kernels.append(hs.HS_LINATTN_CHUNKED_TC)
+    kernels = [hs.HS_LINATTN_SINGLE_TOKEN, hs.HS_LINATTN_RECURRENT, hs.HS_LINATTN_AUTO,
+               hs.HS_LINATTN_CHUNKED_TC]
     q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
     tok_b, tok_f = nH * d * 2, nH * d * 4
     res = []

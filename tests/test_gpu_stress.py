@@ -3,8 +3,8 @@
 Each call (``hs_inputs.gen_stress_case``) draws a random batch, resume points, tail lengths
 and checkpoint interval, then plants stress on random token ranges: growing gates, strong
 gates (-30, -1.2), a zero gate, v scaled by 2^17, q and k scaled by 64, starting states up to
-2^16.  Every kernel that accepts the call (AUTO, the recurrent kernel, the tensor-core kernel
-at d = 128, the single-token kernel for calls of at most one token per problem) must stay
+2^16.  Every kernel that accepts the call (AUTO, the recurrent kernel, the tensor-core
+kernel, the single-token kernel for calls of at most one token per problem) must stay
 within the max-normalised error bound 2e-3 for outputs, final states and checkpoints.
 
 The paper makes numerical control part of the method (Section 4, Table 3): these calls are
@@ -28,9 +28,7 @@ BLOCKS = 12                 # 300 seeds from 200000
 
 
 def _kernels(case):
-    ks = [hs.HS_LINATTN_AUTO, hs.HS_LINATTN_RECURRENT]
-    if case.d == 128:
-        ks.append(hs.HS_LINATTN_CHUNKED_TC)
+    ks = [hs.HS_LINATTN_AUTO, hs.HS_LINATTN_RECURRENT, hs.HS_LINATTN_CHUNKED_TC]
     if max(case.n_tokens) <= 1:
         ks.append(hs.HS_LINATTN_SINGLE_TOKEN)
     return ks
