@@ -108,10 +108,13 @@ def source_hash(kernel: str) -> str:
     return h.hexdigest()[:12]
 
 
+PROFILES = os.path.join(ROOT, "profiles")
+
+
 def _profile_rows(fname, ncols):
     """Rows `kernel v1 .. v_ncols source_hash capture ...` of a profiles/ table whose source
     hash still matches the kernel's source; stale rows map to None."""
-    p = os.path.join(ROOT, "profiles", fname)
+    p = os.path.join(PROFILES, fname)
     out = {}
     if os.path.exists(p):
         for line in open(p):
