@@ -1,15 +1,17 @@
 // Gated linear attention, one token per problem (a decode step):
 //     S' = diag(g) S + k v^T,   o = q S',   g = exp(a).
 //
-// One CTA per (problem, head).  Thread (rg, cg) holds rows [16*rg, 16*rg+16)
-// and columns [4*cg, 4*cg+4) of the d x d float32 state in registers; the
-// lanes of a warp are the column groups, so every state load and store of a
-// warp is whole 512-byte rows.  The token's inputs are read straight from
-// global memory (each row group's q/k/a are one broadcast per warp) before the
-// state (issued in this order the step is 3.0 us instead of 3.2 us on the bench's
-// decode phase), the state goes back to memory as soon as it is updated, and the
-// row groups' partial outputs meet once in shared memory: one block-wide barrier
-// per step.
+// One CTA per (problem, head), d^2/32 threads.  Thread (rg, cg) holds rows
+// [16*rg, 16*rg+16) and columns [2*cg, 2*cg+2) of the d x d float32 state in
+// registers; the lanes of a warp are column groups, so every state load and
+// store of a warp is 256 contiguous bytes of one row.  Two columns per thread
+// measured 2.90 us per bench decode step, against 3.05 us for four columns over
+// half as many threads and 3.16 us for one column over twice as many.  The
+// token's inputs are read straight from global memory (each row group's q/k/a
+// are one broadcast per warp) before the state (issued in this order the step
+// was 3.0 us instead of 3.2 us with four columns per thread), the state goes
+// back to memory as soon as it is updated, and the row groups' partial outputs
+// meet once in shared memory: one block-wide barrier per step.
 //
 // The arithmetic is exactly that of the per-token recurrent kernel and of the
 // short segments of the chunked tensor-core kernel: g = expf(a); every element
@@ -37,9 +39,9 @@ __device__ __forceinline__ float bf16_hi(uint32_t w)
 }
 
 template <int D>
-__global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __grid_constant__ GlaParams p)
+__global__ void __launch_bounds__((D / 2) * (D / 16)) gla_decode_kernel(const __grid_constant__ GlaParams p)
 {
-    constexpr int NCG = D / 4;        // column groups of 4 (lanes)
+    constexpr int NCG = D / 2;        // column groups of 2 (lanes)
     constexpr int NRG = D / 16;       // row groups of 16
     __shared__ __align__(16) float spart[NRG][D];
     const int b = blockIdx.x / p.n_heads;
@@ -68,7 +70,7 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __
     const int64_t row = ((int64_t)p.row0[b]) * p.n_heads + h;   // the call's one token
     const uint4 *q8 = reinterpret_cast<const uint4 *>(p.q + row * D + 16 * rg);
     const uint4 *k8 = reinterpret_cast<const uint4 *>(p.k + row * D + 16 * rg);
-    const uint2 v2 = *reinterpret_cast<const uint2 *>(p.v + row * D + 4 * cg);
+    const uint32_t v2 = *reinterpret_cast<const uint32_t *>(p.v + row * D + 2 * cg);
     uint32_t qw[8], kw[8];
     *reinterpret_cast<uint4 *>(&qw[0]) = q8[0];
     *reinterpret_cast<uint4 *>(&qw[4]) = q8[1];
@@ -76,37 +78,33 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __
     *reinterpret_cast<uint4 *>(&kw[4]) = k8[1];
     // the row group's 16 gates: lane l computes g of row 16 rg + (l mod 16) once, and every
     // lane reads the value it needs from the lane of its half-warp that holds it (the same
-    // expf, so bit-identical).  At d = 128 a warp is one row group (both halves compute the
-    // same 16 values); at d = 64 each half-warp is one row group.
+    // expf, so bit-identical).  A row group spans d/64 warps, so both halves of a warp compute
+    // the same 16 values.
     const int lane = tid & 31;
     const float g_own = expf(p.log_g[row * D + 16 * rg + (lane & 15)]);
 
     float *st = p.state + ((int64_t)b * p.n_heads + h) * D * D;
-    float4 S[16];
+    float2 S[16];
 #pragma unroll
     for (int r = 0; r < 16; ++r)
-        S[r] = *reinterpret_cast<const float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg);
-    const float4 v4 = make_float4(bf16_lo(v2.x), bf16_hi(v2.x), bf16_lo(v2.y), bf16_hi(v2.y));
+        S[r] = *reinterpret_cast<const float2 *>(st + (int64_t)(16 * rg + r) * D + 2 * cg);
+    const float2 vv = make_float2(bf16_lo(v2), bf16_hi(v2));
 
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    float2 acc = make_float2(0.f, 0.f);
 #pragma unroll
     for (int r = 0; r < 16; ++r) {
         const float g = __shfl_sync(0xffffffffu, g_own, (lane & 16) | r);
         const float kk = (r & 1) ? bf16_hi(kw[r >> 1]) : bf16_lo(kw[r >> 1]);
         const float qq = (r & 1) ? bf16_hi(qw[r >> 1]) : bf16_lo(qw[r >> 1]);
-        S[r].x = fmaf(g, S[r].x, kk * v4.x);
-        S[r].y = fmaf(g, S[r].y, kk * v4.y);
-        S[r].z = fmaf(g, S[r].z, kk * v4.z);
-        S[r].w = fmaf(g, S[r].w, kk * v4.w);
+        S[r].x = fmaf(g, S[r].x, kk * vv.x);
+        S[r].y = fmaf(g, S[r].y, kk * vv.y);
         acc.x = fmaf(qq, S[r].x, acc.x);
         acc.y = fmaf(qq, S[r].y, acc.y);
-        acc.z = fmaf(qq, S[r].z, acc.z);
-        acc.w = fmaf(qq, S[r].w, acc.w);
     }
 #pragma unroll
     for (int r = 0; r < 16; ++r)
-        *reinterpret_cast<float4 *>(st + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
-    *reinterpret_cast<float4 *>(&spart[rg][4 * cg]) = acc;
+        *reinterpret_cast<float2 *>(st + (int64_t)(16 * rg + r) * D + 2 * cg) = S[r];
+    *reinterpret_cast<float2 *>(&spart[rg][2 * cg]) = acc;
 
     const int C = p.ckpt_interval;
     if (C > 0 && p.ckpt_slots != nullptr && (pos0 + 1) % C == 0) {
@@ -121,7 +119,7 @@ __global__ void __launch_bounds__((D / 4) * (D / 16)) gla_decode_kernel(const __
             slot += (int64_t)h * D * D;
 #pragma unroll
             for (int r = 0; r < 16; ++r)
-                *reinterpret_cast<float4 *>(slot + (int64_t)(16 * rg + r) * D + 4 * cg) = S[r];
+                *reinterpret_cast<float2 *>(slot + (int64_t)(16 * rg + r) * D + 2 * cg) = S[r];
         }
     }
     __syncthreads();
@@ -141,8 +139,8 @@ cudaError_t launch_gla_decode(const GlaParams &p, int d, cudaStream_t s)
 {
     const unsigned grid = (unsigned)p.batch * (unsigned)p.n_heads;
     if (d == 128)
-        return launch_pdl(gla_decode_kernel<128>, dim3(grid), dim3(256), 0, s, p);
-    return launch_pdl(gla_decode_kernel<64>, dim3(grid), dim3(64), 0, s, p);
+        return launch_pdl(gla_decode_kernel<128>, dim3(grid), dim3(512), 0, s, p);
+    return launch_pdl(gla_decode_kernel<64>, dim3(grid), dim3(128), 0, s, p);
 }
 
 }  // namespace hs
