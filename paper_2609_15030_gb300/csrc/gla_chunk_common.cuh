@@ -52,7 +52,8 @@ constexpr int kPrefetch = 2;                // segments requested into L2 ahead 
 constexpr uint32_t SET_BYTES = 57344;   // one fast operand set:
 constexpr uint32_t S_QH = 0;            //   Q~  fp16 [64 tok i][D]                     16 KiB
 constexpr uint32_t S_KH = 16384;        //   K~  fp16 [64 tok j][D]                     16 KiB
-constexpr uint32_t S_B2H = 32768;       //   [A ; K~^T] fp16 [64 i + D][64 tok j]       24 KiB
+constexpr uint32_t S_AH = 32768;        //   A   fp16 [64 tok i][64 tok j]                8 KiB
+                                        //   (16 KiB after it unused)
 constexpr uint32_t X_QT = 0;            // exact path (over both sets): Q~ tf32 [64][D]         32 KiB
 constexpr uint32_t X_LAM = 32768;       //   Lam f32 [64 tok][D], row-major                     32 KiB
 constexpr uint32_t X_B2 = 65536;        //   [A ; K^^T] tf32 [64 i + D][64 tok j]               48 KiB
@@ -100,10 +101,10 @@ struct Geo {
     static constexpr int TPG = CH / NQ;           // tokens per group: 16 or 8
     static constexpr int CW = D / 2;              // state columns per state thread: 64 or 32
     static constexpr int NG = D / 16;             // short segments: partial sums over 16 key rows
-    static constexpr int ROWS = 64 + D;           // rows of the [A ; K~^T] operands
+    static constexpr int ROWS = 64 + D;           // rows of the exact path's [A ; K^^T] operand
     static constexpr uint32_t O1 = TM_S + D;      // D_O of odd chunks, right of S^T
     static constexpr uint32_t SHI = TM_S + D;     // exact path: hi part of S^T
-    static constexpr uint32_t IDF_UPD = idesc_f16(128, 64 + D);    // [D_O | S^T] += V^T [..]^T
+    static constexpr uint32_t IDF_ST = idesc_f16(128, D, 1);       // S^T += V^T K~ (K~ read MN-major)
     static constexpr uint32_t IDT_ST = idesc_tf32(128, D, 0, 0);   // exact: S^T += V^T K^
     static constexpr uint32_t STAGE = 3 * CH * D * 2 + CH * D * 4;  // staged q, k, v, log-gates
 };
@@ -332,19 +333,15 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
         lam_ok = t0 >= -kLamRange && t1 >= -kLamRange;
     }
     uint8_t *set = smem + par * SET_BYTES;
-    const int rowK = par ? 0 : 64;
     __nv_bfloat162 bq = __float2bfloat162_rn(0.f), bk = bq;   // max |q|, |k|
     __half2 hq = __float2half2_rn(0.f), hk = hq;                 // max |Q~|, |K~| (fp16)
-    // runs of 8 tokens; within a run, token pairs: Q~ and K~ as fp16 pairs of key dims,
-    // K~^T rows 2dp and 2dp+1 as fp16 pairs of tokens (byte permutes of the K~ pairs)
+    // runs of 8 tokens; within a run, token pairs: Q~ and K~ as fp16 pairs of key dims
     float *sDg = reinterpret_cast<float *>(smem + OFF_DG) + par * 128 + (dp >> 5) * 64;
 #pragma unroll 1
     for (int grp = 0; grp < G::TPG / 8; ++grp) {
-        uint32_t kt0[4], kt1[4];
         float pd[8];   // q . k over this thread's two key dims, tokens 8 grp + 0..7 of its group
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
-            uint32_t kp[2];
 #pragma unroll
             for (int t = 0; t < 2; ++t) {
                 const int i = G::TPG * qt + 8 * grp + 2 * u + t;
@@ -356,28 +353,20 @@ __device__ __forceinline__ void build_fast(uint8_t *smem, uint32_t tmem, int L, 
                 const float q0 = __uint_as_float(q2 << 16), q1 = __uint_as_float(q2 & 0xFFFF0000u);
                 const float k0 = __uint_as_float(k2 << 16), k1 = __uint_as_float(k2 & 0xFFFF0000u);
                 const uint32_t qp = pack_h2(q0 * ex2(run0), q1 * ex2(run1));
-                kp[t] = pack_h2(k0 * ex2(-run0), k1 * ex2(-run1));
+                const uint32_t kp = pack_h2(k0 * ex2(-run0), k1 * ex2(-run1));
                 pd[2 * u + t] = fmaf(q1, k1, q0 * k0);
                 *reinterpret_cast<uint32_t *>(set + S_QH + h_off(64, i, 2 * dp)) = qp;
-                *reinterpret_cast<uint32_t *>(set + S_KH + h_off(64, i, 2 * dp)) = kp[t];
+                *reinterpret_cast<uint32_t *>(set + S_KH + h_off(64, i, 2 * dp)) = kp;
                 bq = bmax_abs(bq, q2);
                 bk = bmax_abs(bk, k2);
                 hq = hmax_abs(hq, qp);
-                hk = hmax_abs(hk, kp[t]);
+                hk = hmax_abs(hk, kp);
             }
-            kt0[u] = __byte_perm(kp[0], kp[1], 0x5410);   // key dim 2dp: tokens (2u, 2u+1)
-            kt1[u] = __byte_perm(kp[0], kp[1], 0x7632);   // key dim 2dp+1
         }
         const int j0 = G::TPG * qt + 8 * grp;
-        {
-            const float dsum = warp_sum8(pd, lane);
-            if ((lane & 3) == 0)
-                sDg[j0 + ((lane >> 2) & 7)] = dsum;
-        }
-        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(G::ROWS, rowK + 2 * dp, j0)) =
-            make_uint4(kt0[0], kt0[1], kt0[2], kt0[3]);
-        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(G::ROWS, rowK + 2 * dp + 1, j0)) =
-            make_uint4(kt1[0], kt1[1], kt1[2], kt1[3]);
+        const float dsum = warp_sum8(pd, lane);
+        if ((lane & 3) == 0)
+            sDg[j0 + ((lane >> 2) & 7)] = dsum;
     }
     // V^T: thread (e, half) packs tokens [32 half, 32 half + 32) of value dim e
     __nv_bfloat162 bv = __float2bfloat162_rn(0.f);
@@ -483,8 +472,8 @@ __device__ __forceinline__ void state_pass(uint8_t *smem, uint32_t tmem, int gpa
 }
 
 
-// ---- the causally masked intra-chunk matrix A (D_A) -> rows rowA.. of set par's [A ; K~^T]
-// (state warps of TMEM lane quarters 0 and 1)
+// ---- the causally masked intra-chunk matrix A (D_A) -> set par's A operand (state warps of
+// TMEM lane quarters 0 and 1)
 template <int D>
 __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
 {
@@ -496,7 +485,6 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
         return;
     const int i = (warp & 3) * 32 + lane;      // TMEM lane = query row
     const int jb = ((warp >> 2) & 1) * 32;      // this warp's 32 key columns
-    const int rowA = par ? D : 0;
     float r[32];
     tmem_ld32(tmem + lrow + (par ? TM_A1 : TM_A0) + jb, r);
     // the diagonal from the builders' float32 partials (one per 64 key dims)
@@ -514,7 +502,7 @@ __device__ __forceinline__ void a_build(uint8_t *smem, uint32_t tmem, int par)
             const float x1 = j0 + 1 == i ? dg : (j0 + 1 <= i ? r[8 * c + 2 * u + 1] : 0.f);
             w[u] = pack_h2(x0, x1);
         }
-        *reinterpret_cast<uint4 *>(set + S_B2H + h_off(Geo<D>::ROWS, rowA + i, jb + 8 * c)) =
+        *reinterpret_cast<uint4 *>(set + S_AH + h_off(64, i, jb + 8 * c)) =
             make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
@@ -809,17 +797,22 @@ __device__ __forceinline__ void fast_issue_sq(uint32_t tmem, uint32_t sb, int pa
     }
 }
 
-// [D_O | S^T] += V^T [A ; K~^T]^T as one N = 64 + D product (even sets order the operand's
-// rows [A ; K~^T] with D_O0 on the left of S^T, odd sets [K~^T ; A] with D_O1 on the right)
+// D_O += V^T A^T and S^T += V^T K~, 16 tokens per step.  K~ is stored token-major for D_A
+// (K-major there, K = key dim); read with N = key dim contiguous it is the MN-major B operand
+// of the state update: 64-dim blocks 8 KiB apart (leading byte offset), 8-token row groups
+// 1 KiB apart (stride byte offset), 16 tokens = 2 KiB per step.
 template <int D>
 __device__ __forceinline__ void fast_issue_update(uint32_t tmem, uint32_t sb, int par)
 {
     const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
     const uint32_t vt = tmem + TM_V + 32 * par;
 #pragma unroll 1
-    for (int kk = 0; kk < CH / 16; ++kk)
-        mma_f16_ts(tmem + (par ? TM_S : TM_O0), vt + kk * 8,
-                   sdesc_sw128(setb + S_B2H + kk * 32, 16, 1024), Geo<D>::IDF_UPD, 1);
+    for (int kk = 0; kk < CH / 16; ++kk) {
+        mma_f16_ts(tmem + (par ? Geo<D>::O1 : TM_O0), vt + kk * 8,
+                   sdesc_sw128(setb + S_AH + kk * 32, 16, 1024), IDF_N64, 1);
+        mma_f16_ts(tmem + TM_S, vt + kk * 8, sdesc_sw128(setb + S_KH + kk * 2048, 8192, 1024),
+                   Geo<D>::IDF_ST, 1);
+    }
 }
 
 // ---- short segments (<= kShort tokens): the per-token recurrence with the recurrent kernel's

@@ -240,10 +240,11 @@ __device__ __forceinline__ void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uin
         : "memory");
 }
 
-// Instruction descriptor, kind::f16 with fp16 A and B (format 0) and an fp32 accumulator.
-__host__ __device__ constexpr uint32_t idesc_f16(int M, int N)
+// Instruction descriptor, kind::f16 with fp16 A and B (format 0) and an fp32 accumulator;
+// b_mn = 1 reads B as MN-major (N contiguous in shared memory) instead of K-major.
+__host__ __device__ constexpr uint32_t idesc_f16(int M, int N, int b_mn = 0)
 {
-    return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+    return (1u << 4) | ((uint32_t)b_mn << 16) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
 __device__ __forceinline__ void tmem_wait_ld()
