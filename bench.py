@@ -92,18 +92,34 @@ KERNEL_SRC = {"gla_decode_kernel": "gla_decode.cu", "gla_chunked_tc_kernel": "gl
 DTYPE = "bf16 q/k/v, fp32 log-gates; fp16 (fast) or tf32 (exact) MMA operands, fp32 accumulate, state and outputs"
 
 
-def source_hash(kernel: str) -> str:
-    """First 12 hex digits of the SHA-256 of the kernel's source file, then the library's
-    internal headers and the public header (what its machine code depends on): a profile row
-    captured under another hash describes another kernel."""
-    import hashlib
+def source_files(kernel: str) -> list:
+    """The kernel's source file and every local header it includes, directly or through
+    other headers (in breadth-first order)."""
+    import re
     name = kernel.split("@")[0].split("<")[0]
-    csrc = os.path.join(ROOT, "paper_2609_15030_gb300", "csrc")
-    files = [os.path.join(csrc, KERNEL_SRC[name])]
-    files += sorted(os.path.join(csrc, f) for f in os.listdir(csrc) if f.endswith(".cuh"))
-    files.append(os.path.join(ROOT, "include", "hs.h"))
+    dirs = [os.path.join(ROOT, "paper_2609_15030_gb300", "csrc"), os.path.join(ROOT, "include")]
+    files, todo = [], [os.path.join(dirs[0], KERNEL_SRC[name])]
+    while todo:
+        f = todo.pop(0)
+        if f in files:
+            continue
+        files.append(f)
+        for inc in re.findall(r'^\s*#\s*include\s+"([^"]+)"', open(f).read(), re.M):
+            for d in dirs:
+                cand = os.path.join(d, inc)
+                if os.path.exists(cand):
+                    todo.append(cand)
+                    break
+    return files
+
+
+def source_hash(kernel: str) -> str:
+    """First 12 hex digits of the SHA-256 of the kernel's source files (`source_files`: what
+    its machine code depends on): a profile row captured under another hash describes
+    another kernel."""
+    import hashlib
     h = hashlib.sha256()
-    for f in files:
+    for f in source_files(kernel):
         h.update(open(f, "rb").read())
     return h.hexdigest()[:12]
 

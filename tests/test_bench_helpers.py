@@ -25,6 +25,18 @@ def test_source_hash_names_the_kernel_source():
     assert h != bench.source_hash("slot_copy_kernel")
 
 
+def test_source_files_follow_the_include_graph():
+    base = lambda k: [os.path.basename(f) for f in bench.source_files(k)]
+    tc, dec = base("gla_chunked_tc_kernel"), base("gla_decode_kernel<128>")
+    assert tc[0] == "gla_chunked_tc.cu" and dec[0] == "gla_decode.cu"
+    for h in ("gla_chunk_common.cuh", "sm100_ptx.cuh", "hs_internal.cuh", "hs.h"):
+        assert h in tc
+    # the decode kernel's hash does not move when only the prefill's headers change
+    assert "gla_chunk_common.cuh" not in dec and "sm100_ptx.cuh" not in dec
+    assert "hs_internal.cuh" in dec and "hs.h" in dec
+    assert base("kv_gather_kernel") == base("kv_scatter_kernel")
+
+
 def test_stale_profile_rows_read_as_null(tmp_path, monkeypatch):
     fresh = bench.source_hash("gla_decode_kernel")
     (tmp_path / "dram_traffic.txt").write_text(
