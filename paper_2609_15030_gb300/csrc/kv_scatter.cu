@@ -104,8 +104,23 @@ kv_gather_kernel(const void *const *cache, void *const *staging, int32_t n_layer
 // [col_off, col_off + col_bytes) of each row (one tensor-parallel rank's heads).
 // The staging page holds the rows' slices back to back (rows * col_bytes bytes).
 // cache <- staging when kGather is false, staging <- cache when it is true.
-template <bool kGather>
-__global__ void __launch_bounds__(kThreads)
+// A slice is small (8 KiB for one FP8 rank of four), so the loads of a unit's block id
+// and layer pointers, which its data loads depend on, cost about as much as its data:
+// each CTA requests the next unit's while it moves the current one.  Slices of at most
+// 2 x 256 vectors take the kU = 2 instantiation, 32 registers and 8 resident CTAs per SM
+// (twice the bytes in flight), larger ones kU = 4.  Measured on 48 x 256 FP8 slices of 8 KiB
+// (one box): 0.60 of the HBM copy peak before (each unit waiting for its own metadata, eight
+// vectors per thread, 4 CTAs per SM), 0.62 with the metadata ahead, 0.72 with kU = 2 at 8 CTAs
+// per SM; 16 and 32 KiB slices: 0.86 and 0.94 with kU = 4, 0.84 and 0.91 with kU = 2.
+struct SliceUnit {
+    const uint8_t *src;
+    uint8_t *dst;
+    int32_t j;     // page index (staging slot)
+    int32_t blk;   // cache block
+};
+
+template <bool kGather, int kU, int kMinBlocks>
+__global__ void __launch_bounds__(kThreads, kMinBlocks)
 kv_slices_kernel(const void *const *from, void *const *to, int32_t n_layers, const int32_t *bt,
                  int32_t n_pages, int64_t page_bytes, int32_t rows, int64_t row_bytes,
                  int64_t col_off, int32_t col_vecs, int64_t num_blocks, int32_t *d_err)
@@ -113,56 +128,73 @@ kv_slices_kernel(const void *const *from, void *const *to, int32_t n_layers, con
     pdl_wait_and_release();
     const int64_t units = (int64_t)n_layers * n_pages;
     const int32_t vecs = rows * col_vecs;                      // 16-byte vectors per page slice
-    for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
+    auto unit = [&](int64_t u) -> SliceUnit {
+        SliceUnit m;
         const int32_t l = (int32_t)(u / n_pages);
-        const int32_t j = (int32_t)(u - (int64_t)l * n_pages);
-        const uint8_t *src = static_cast<const uint8_t *>(from[l]);
-        uint8_t *dst = static_cast<uint8_t *>(to[l]);
-        const int32_t blk = bt[j];
+        m.j = (int32_t)(u - (int64_t)l * n_pages);
+        m.src = static_cast<const uint8_t *>(from[l]);
+        m.dst = static_cast<uint8_t *>(to[l]);
+        m.blk = bt[m.j];
+        return m;
+    };
+    int64_t u = blockIdx.x;
+    SliceUnit cur;
+    if (u < units)
+        cur = unit(u);
+    while (u < units) {
+        const int64_t un = u + gridDim.x;
+        SliceUnit nxt = cur;
+        if (un < units)
+            nxt = unit(un);   // in flight while this unit moves
+        const uint8_t *src = cur.src;
+        uint8_t *dst = cur.dst;
+        bool ok = true;
         if (src == nullptr || dst == nullptr) {
             if (threadIdx.x == 0)
                 report(d_err, HS_DEVERR_NULL);
-            continue;
-        }
-        if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u) != 0) {
+            ok = false;
+        } else if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15u) != 0) {
             if (threadIdx.x == 0)
                 report(d_err, HS_DEVERR_MISALIGNED);
-            continue;
-        }
-        if (blk < 0 || (int64_t)blk >= num_blocks) {
+            ok = false;
+        } else if (cur.blk < 0 || (int64_t)cur.blk >= num_blocks) {
             if (threadIdx.x == 0)
                 report(d_err, HS_DEVERR_BLOCK_OOB);
-            continue;
+            ok = false;
         }
-        const uint8_t *cache_page = (kGather ? src : dst) + (int64_t)blk * page_bytes + col_off;
-        const int64_t stage_page = (int64_t)j * vecs * 16;
-        for (int32_t base = threadIdx.x; base < vecs; base += kThreads * kUnroll) {
-            uint4 r[kUnroll];
-            int64_t coff[kUnroll];     // byte offset of the vector in the cache page
+        if (ok) {
+            const uint8_t *cache_page = (kGather ? src : dst) + (int64_t)cur.blk * page_bytes + col_off;
+            const int64_t stage_page = (int64_t)cur.j * vecs * 16;
+            for (int32_t base = threadIdx.x; base < vecs; base += kThreads * kU) {
+                uint4 r[kU];
+                int64_t coff[kU];     // byte offset of the vector in the cache page
 #pragma unroll
-            for (int x = 0; x < kUnroll; ++x) {
-                const int32_t i = base + x * kThreads;
-                const int32_t row = i / col_vecs;
-                coff[x] = (int64_t)row * row_bytes + (int64_t)(i - row * col_vecs) * 16;
-                if (i < vecs) {
-                    const uint8_t *s = kGather ? cache_page + coff[x] : src + stage_page + (int64_t)i * 16;
-                    r[x] = ld_stream(reinterpret_cast<const uint4 *>(s));
+                for (int x = 0; x < kU; ++x) {
+                    const int32_t i = base + x * kThreads;
+                    const int32_t row = i / col_vecs;
+                    coff[x] = (int64_t)row * row_bytes + (int64_t)(i - row * col_vecs) * 16;
+                    if (i < vecs) {
+                        const uint8_t *sp = kGather ? cache_page + coff[x] : src + stage_page + (int64_t)i * 16;
+                        r[x] = ld_stream(reinterpret_cast<const uint4 *>(sp));
+                    }
+                }
+#pragma unroll
+                for (int x = 0; x < kU; ++x) {
+                    const int32_t i = base + x * kThreads;
+                    if (i < vecs) {
+                        uint8_t *dp = kGather ? dst + stage_page + (int64_t)i * 16
+                                              : const_cast<uint8_t *>(cache_page) + coff[x];
+                        st_stream(reinterpret_cast<uint4 *>(dp), r[x]);
+                    }
                 }
             }
-#pragma unroll
-            for (int x = 0; x < kUnroll; ++x) {
-                const int32_t i = base + x * kThreads;
-                if (i < vecs) {
-                    uint8_t *d = kGather ? dst + stage_page + (int64_t)i * 16
-                                         : const_cast<uint8_t *>(cache_page) + coff[x];
-                    st_stream(reinterpret_cast<uint4 *>(d), r[x]);
-                }
-            }
         }
+        cur = nxt;
+        u = un;
     }
 }
 
-// 8 resident CTAs of 256 threads per SM; at most 4 waves, never more CTAs than units
+// up to 8 resident CTAs of 256 threads per SM; at most 4 waves of 8, never more CTAs than units
 int64_t kv_grid(int32_t n_layers, int32_t n_pages, int sm_count)
 {
     const int64_t units = (int64_t)n_layers * n_pages;
@@ -188,13 +220,12 @@ cudaError_t launch_kv_slices(bool gather, const void *const *from, void *const *
 {
     const int64_t grid = kv_grid(n_layers, n_pages, sm_count);
     const int64_t row_bytes = page_bytes / rows;
-    if (gather)
-        return launch_pdl(kv_slices_kernel<true>, dim3((unsigned)grid), dim3(kThreads), 0, s, from,
-                          to, n_layers, bt, n_pages, page_bytes, rows, row_bytes, col_off,
-                          (int32_t)(col_bytes / 16), num_blocks, d_err);
-    return launch_pdl(kv_slices_kernel<false>, dim3((unsigned)grid), dim3(kThreads), 0, s, from, to,
-                      n_layers, bt, n_pages, page_bytes, rows, row_bytes, col_off,
-                      (int32_t)(col_bytes / 16), num_blocks, d_err);
+    const int32_t col_vecs = (int32_t)(col_bytes / 16);
+    const bool small = (int64_t)rows * col_vecs <= 2 * kThreads;
+    auto kern = gather ? (small ? kv_slices_kernel<true, 2, 8> : kv_slices_kernel<true, 4, 1>)
+                       : (small ? kv_slices_kernel<false, 2, 8> : kv_slices_kernel<false, 4, 1>);
+    return launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), 0, s, from, to, n_layers, bt, n_pages,
+                      page_bytes, rows, row_bytes, col_off, col_vecs, num_blocks, d_err);
 }
 
 cudaError_t launch_kv_scatter(const void *const *staging, void *const *cache, int32_t n_layers,

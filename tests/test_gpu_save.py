@@ -241,3 +241,38 @@ def test_rank_slices_with_a_row_split_that_does_not_divide_the_block():
     got = cache.cpu().numpy()
     for l in range(L):
         assert np.array_equal(got[l], want[l])
+
+
+@pytest.mark.parametrize("rows,row_bytes,off,cb", [
+    (32, 2048, 1024, 1024),   # bf16 pages, two ranks: 2,048 vectors per slice (wide instantiation)
+    (33, 1024, 256, 256),     # 528 vectors: just past the narrow instantiation's limit
+    (32, 1024, 512, 256),     # 512 vectors: the narrow one's largest slice
+    (1, 8192, 0, 8192),       # one contiguous 8 KiB row per page
+])
+def test_rank_slices_of_every_width_round_trip(rows, row_bytes, off, cb):
+    """Slices on either side of the launch's choice between its narrow (at most 512 vectors per
+    slice, eight CTAs per SM) and wide instantiations: the restore matches the oracle's slice
+    scatter into a poisoned cache and the save gives the staging back bit for bit."""
+    dev = device()
+    L, nb, n_pages = 3, 40, 17
+    P = rows * row_bytes
+    rng = np.random.default_rng(rows * 7 + cb)
+    st = torch.from_numpy(rng.integers(0, 256, size=(L, n_pages * rows * cb), dtype=np.uint8)).to(dev)
+    cache = torch.full((L, nb * P), POISON, dtype=torch.uint8, device=dev)
+    bt = torch.from_numpy(gen_block_table(25, rows, n_pages, nb)).to(dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    cp = hs.ptr_array([cache[l] for l in range(L)], dev)
+    hs.hs_restore_kv_page_slices(hs.ptr_array([st[l] for l in range(L)], dev), cp, L, bt, n_pages,
+                                 P, rows, off, cb, nb, err)
+    back = torch.zeros_like(st)
+    hs.hs_save_kv_page_slices(cp, hs.ptr_array([back[l] for l in range(L)], dev), L, bt, n_pages,
+                              P, rows, off, cb, nb, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    assert torch.equal(back, st)
+    want = [np.full(nb * P, POISON, np.uint8) for _ in range(L)]
+    oracle.scatter_slices([st[l].cpu().numpy() for l in range(L)], want, bt.cpu().numpy(), n_pages,
+                          P, rows, off, cb)
+    got = cache.cpu().numpy()
+    for l in range(L):
+        assert np.array_equal(got[l], want[l]), l
