@@ -1383,10 +1383,12 @@ def run_long(dev, reps=3, quiet=False):
             shape_t = hs.make_shape(B, nH, d, d, Lmax)
             slot_ptrs = hs.ptr_array([slots[b] for b in range(B)], dev) if L % C == 0 else None
             tok = c * nH * d
-            def resume():
+            def resume(mid=None):
                 for b in range(B):      # the batch's states ride with the first request's pages
                     hs.hs_restore_request(stg_ptrs[b], cache_ptrs, nF, bts[b], n_pages, pb, NB,
                                           src_ptrs, dst_ptrs, nL if b == 0 else 0, B * nH * d * d)
+                if mid is not None:
+                    mid.record()
                 for l in range(nL):
                     hs.hs_linattn_prefill_from_state(
                         shape_t, q.data_ptr() + 2 * tok, k.data_ptr() + 2 * tok, v.data_ptr() + 2 * tok,
@@ -1396,37 +1398,53 @@ def run_long(dev, reps=3, quiet=False):
             ckp = hs.ptr_array([slots[b * nck + m] for b in range(B) for m in range(per)], dev)
             if hs.hs_linattn_num_checkpoints([c] * B, [tail] * B, C) != (B if L % C == 0 else 0):
                 raise SystemExit("unexpected checkpoint count")
-            def recompute():
+            def recompute(mid=None):
                 for l in range(nL):
                     states[l].zero_()
                     hs.hs_linattn_prefill_from_state(shape_t, q, k, v, a, o, states[l], [0] * B, [L] * B, C, ckp)
+                if mid is not None:
+                    mid.record()
                 for b in range(B):
                     hs.hs_restore_kv_pages(stg_ptrs[b], cache_ptrs, nF, bts[b], L // P, pb, NB)
-            res = {}
+            res, part = {}, {}
             for nm, fn in (("resume", resume), ("recompute", recompute)):
                 fn()
                 torch.cuda.synchronize(dev)
-                ts = []
+                ts, t1s = [], []
                 for _ in range(reps):
-                    e0, e1 = ev(), ev()
+                    e0, em, e1 = ev(), ev(), ev()
                     e0.record()
-                    fn()
-                    e1.record()
+                    fn(em)       # an event between the arm's two parts (restore | prefills,
+                    e1.record()  # prefills | KV write)
                     torch.cuda.synchronize(dev)
                     ts.append(e0.elapsed_time(e1))
+                    t1s.append(e0.elapsed_time(em))
                 res[nm] = statistics.median(ts)
+                part[nm] = statistics.median(t1s)
             # algorithmic bytes of each arm: resume = KV restore of [0,c) + state restore +
             # the tail prefill of every linear layer; recompute = the prefill of [0,L) of every
             # linear layer emitting every checkpoint + the KV write of L tokens
-            b_res = (B * kv_bytes(nF, n_pages, pb) + 2 * nL * B * nH * d * d * 4
-                     + nL * gla_bytes(B, nH, d, tail, 1 if L % C == 0 else 0))
-            b_rec = nL * gla_bytes(B, nH, d, L, L // C) + B * kv_bytes(nF, L // P, pb)
+            b_restore = B * kv_bytes(nF, n_pages, pb) + 2 * nL * B * nH * d * d * 4
+            b_tail = nL * gla_bytes(B, nH, d, tail, 1 if L % C == 0 else 0)
+            b_res = b_restore + b_tail
+            b_k2 = nL * gla_bytes(B, nH, d, L, L // C)
+            b_rec = b_k2 + B * kv_bytes(nF, L // P, pb)
             peak = _peaks()[0]
+            frac = lambda nb, ms: round(nb / (ms * 1e-3) / 1e9 / peak, 3)
             row = {"L": L, "hit": hit, "c": c, "tail": tail, "ttft_resume_ms": round(res["resume"], 3),
                    "ttft_recompute_ms": round(res["recompute"], 3),
                    "ratio": round(res["recompute"] / res["resume"], 1),
                    "resume_hbm_frac": round(b_res / (res["resume"] * 1e-3) / 1e9 / peak, 3),
-                   "recompute_hbm_frac": round(b_rec / (res["recompute"] * 1e-3) / 1e9 / peak, 3)}
+                   "recompute_hbm_frac": round(b_rec / (res["recompute"] * 1e-3) / 1e9 / peak, 3),
+                   # the arms' parts (events between them): K1 + K2a, the restore of 6
+                   # attention layers' pages and 18 states for the batch; K2, the 512-token
+                   # tails of the 18 linear layers; K2 over [0,L) emitting every checkpoint
+                   "restore_ms": round(part["resume"], 3),
+                   "restore_hbm_frac": frac(b_restore, part["resume"]),
+                   "k2_tail_ms": round(res["resume"] - part["resume"], 3),
+                   "k2_tail_hbm_frac": frac(b_tail, res["resume"] - part["resume"]),
+                   "k2_recompute_ms": round(part["recompute"], 3),
+                   "k2_recompute_hbm_frac": frac(b_k2, part["recompute"])}
             rows.append(row)
             if not quiet:
                 print(json.dumps(row), flush=True)
