@@ -992,6 +992,70 @@ def sweep_run(dev, reps=10):
             "rows": rows}
 
 
+def packed_run(dev, reps=10):
+    """Packed varlen tails: the tails of one engine batch back to back without padding, each
+    problem with its own resume point, in one launch (hs_linattn_prefill_packed).  The batch
+    is the hybrid workload's nine requests x nine linear layers (81 problems, 16 heads, d = 128,
+    C = 256) with seeded tail lengths in [65, 512] and resume points on the 256-token grid in
+    [0, 4352]; the checkpoints each tail crosses are emitted.  Timed alone between CUDA events
+    with L2 flushed before each call, median of `reps`; against the same problems in the padded
+    layout (rows of 512 tokens)."""
+    import numpy as np
+    import torch
+    import paper_2609_15030_gb300 as hs
+    from hs_inputs import torch_gen_linear
+    nP, nH, d, C, Tmax = HYBRID12.n_lin * N_REQ, HYBRID12.n_heads, HYBRID12.d, HYBRID12.ckpt, 512
+    rng = np.random.default_rng(21)
+    n_tok = [int(x) for x in rng.integers(65, Tmax + 1, nP)]
+    pos0 = [int(x) * C for x in rng.integers(0, 18, nP)]
+    cu = np.concatenate([[0], np.cumsum(n_tok)]).astype(np.int64)
+    rows = int(cu[-1])
+    q, k, v, a = torch_gen_linear(13, 0, 1, rows, nH, d, dev)
+    o = torch.empty((rows, nH, d), device=dev)
+    qp, kp, vp, ap = (torch_gen_linear(13, 0, nP, Tmax, nH, d, dev))
+    op = torch.empty((nP, Tmax, nH, d), device=dev)
+    st0 = torch.randn((nP, nH, d, d), device=dev,
+                      generator=torch.Generator(device=dev).manual_seed(14)) * 0.5
+    state = torch.empty_like(st0)
+    nck = hs.hs_linattn_num_checkpoints(pos0, n_tok, C)
+    slots = torch.empty((max(nck, 1), nH, d, d), device=dev)
+    sp = hs.ptr_array([slots[i] for i in range(nck)], dev) if nck else None
+    stream = torch.cuda.current_stream(dev)
+    shape_p = hs.make_shape(nP, nH, d, d, 0)
+    shape_d = hs.make_shape(nP, nH, d, d, Tmax)
+
+    def packed():
+        hs.hs_linattn_prefill_packed(shape_p, q, k, v, a, o, state, pos0, n_tok, cu.tolist(), C, sp,
+                                     None, stream.cuda_stream)
+
+    def padded():
+        hs.hs_linattn_prefill_from_state(shape_d, qp, kp, vp, ap, op, state, pos0, n_tok, C, sp, None,
+                                         stream.cuda_stream)
+    res = {}
+    for nm, fn in (("packed", packed), ("padded", padded)):
+        ts = []
+        for i in range(reps + 2):
+            state.copy_(st0)
+            _l2_flush(torch, dev)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize(dev)
+            if i >= 2:
+                ts.append(e0.elapsed_time(e1) * 1e3)
+        res[nm] = statistics.median(ts)
+    nb = sum(gla_bytes(1, nH, d, n, (p0 + n) // C - p0 // C) for p0, n in zip(pos0, n_tok))
+    peak = _peaks()[0]
+    return {"problems": nP, "tokens": rows, "tail_min": min(n_tok), "tail_max": max(n_tok),
+            "checkpoints": nck, "packed_us": round(res["packed"], 2),
+            "packed_tokens_per_s": round(rows / (res["packed"] * 1e-6), 1),
+            "packed_hbm_frac": round(nb / (res["packed"] * 1e-6) / 1e9 / peak, 4),
+            "padded_us": round(res["padded"], 2),
+            "timing": "each call alone, L2 flushed before it, median of %d" % reps}
+
+
 def tiny_run(dev, reps=20):
     """Tiny hybrid stack (1 linear layer: 2 heads, d = 64, C = 64; 1 full layer: 2 KV heads,
     head_dim 64, page 16), seed 0, N = 256, complete hit -> c = 192: the resumed request
@@ -1613,6 +1677,8 @@ def main():
             out["ttft_us"] = ttft_arms(wl)
         with _nvtx("tiny stack latency"):
             out["tiny_latency"] = tiny_run(dev)
+        with _nvtx("packed varlen tails"):
+            out["packed_tails"] = packed_run(dev)
         with _nvtx("single-layer sweep"):
             out["sweep"] = sweep_run(dev)
         red = [1.0 - r["resume_us"] / r["recompute_us"] for r in out["ttft_us"].values()]
