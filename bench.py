@@ -914,12 +914,13 @@ def _l2_flush(torch, dev, buf=[]):
     buf[0].fill_(1)
 
 
-def sweep_run(dev, reps=10):
+def sweep_run(dev, reps=10, scan=True):
     """Single-layer kernel sweep: one linear layer, 16 heads, d = 128, checkpoints every 512,
     batch 1.  For each L in 512..4608: the resumed tail prefill (c = C floor((L-1)/C), 512
     tokens from the state at c, emitting the checkpoint at L; the hit L-37 aligns to the same
-    c) and the recomputation of [0,L) from the zero state emitting every checkpoint.  Each
-    call is timed alone between CUDA events with L2 flushed before it; median of `reps`."""
+    c) and the recomputation of [0,L) from the zero state emitting every checkpoint; with
+    `scan`, both also through the segment-parallel prefill.  Each call is timed alone between
+    CUDA events with L2 flushed before it; median of `reps`."""
     import torch
     import paper_2609_15030_gb300 as hs
     from hs_inputs import SWEEP, torch_gen_linear
@@ -936,6 +937,8 @@ def sweep_run(dev, reps=10):
     tb, tbf = nH * d * 2, nH * d * 4
     peak = _peaks()[0]
     tensor = _tensor_pipe()
+    ws_bytes = hs.hs_linattn_scan_workspace_bytes(shape, [0], [Lmax])
+    ws = torch.empty((ws_bytes // 4,), device=dev)
     rows = []
     for L in SWEEP_LENGTHS:
         c, _, tail = hs.hs_align_prefix(L, L, list(range(C, L + 1, C)), S.page)
@@ -953,9 +956,24 @@ def sweep_run(dev, reps=10):
         def recompute():
             hs.hs_linattn_prefill_from_state(shape, q, k, v, a, o, state, [0], [L], C, rec_ptrs,
                                              None, stream.cuda_stream)
+
+        # the same two calls through the segment-parallel prefill (its own workspace)
+        def resume_scan():
+            hs.hs_linattn_prefill_scan(
+                shape, q.data_ptr() + c * tb, k.data_ptr() + c * tb, v.data_ptr() + c * tb,
+                a.data_ptr() + c * tbf, o.data_ptr() + c * tbf, state, [c], [tail], C, tail_ptrs,
+                ws, ws_bytes, None, stream.cuda_stream)
+
+        def recompute_scan():
+            hs.hs_linattn_prefill_scan(shape, q, k, v, a, o, state, [0], [L], C, rec_ptrs, ws,
+                                       ws_bytes, None, stream.cuda_stream)
         res = {}
-        for nm, fn, init in (("tail", resume, lambda: state.copy_(ck)),
-                             ("recompute", recompute, lambda: state.zero_())):
+        arms = [("tail", resume, lambda: state.copy_(ck)),
+                ("recompute", recompute, lambda: state.zero_())]
+        if scan:
+            arms += [("tail_scan", resume_scan, lambda: state.copy_(ck)),
+                     ("recompute_scan", recompute_scan, lambda: state.zero_())]
+        for nm, fn, init in arms:
             ts = []
             for i in range(reps + 2):
                 init()
@@ -983,9 +1001,19 @@ def sweep_run(dev, reps=10):
             "recompute_tokens_per_s": round(L / res["recompute"], 1),
             "recompute_hbm_frac": round(b_rec / res["recompute"] / 1e9 / peak, 4),
             "recompute_tensor_pipe": tp_r["active"] if tp_r else None})
-    del q, k, v, a, o, slots
+        if scan:
+            rows[-1].update({
+                "tail_scan_us": round(res["tail_scan"] * 1e6, 2),
+                "tail_scan_hbm_frac": round(b_tail / res["tail_scan"] / 1e9 / peak, 4),
+                "recompute_scan_us": round(res["recompute_scan"] * 1e6, 2),
+                "recompute_scan_hbm_frac": round(b_rec / res["recompute_scan"] / 1e9 / peak, 4)})
+    del q, k, v, a, o, slots, ws
     return {"workload": "single-layer sweep: 16 heads, d = 128, C = 512, batch 1, tails of 512 "
                         "(complete hit and hit L-37 align to the same c)",
+            "scan": "*_scan_*: the same calls through hs_linattn_prefill_scan (every 64-token "
+                    "segment its own tensor-core problem from the zero state, an elementwise "
+                    "state scan, every segment again from its start state; algorithmic bytes "
+                    "as the sequential call's)",
             "timing": f"each call alone, L2 flushed before it, median of {reps}",
             "tensor_pipe": "sm__pipe_tensor_cycles_active, % of active cycles, from the committed "
                            "ncu capture of `bench.py --case sweep` (null when the kernel changed since)",
@@ -1392,7 +1420,7 @@ def run_case(name: str, iters: int = 5):
     elif name == "sweep":
         # single-layer sweep: each L's 512-token tail from c, then its recomputation of [0,L),
         # one call each with L2 flushed before it (18 prefill launches, L = 512 .. 4608)
-        r = sweep_run(dev, reps=1)
+        r = sweep_run(dev, reps=1, scan=False)
         for row in r["rows"]:
             print(json.dumps({k: row[k] for k in ("L", "tail_us", "recompute_us")}), flush=True)
     else:

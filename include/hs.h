@@ -370,6 +370,56 @@ hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t 
                                     int32_t *d_err, cudaStream_t stream);
 
 /*
+ * hs_linattn_prefill_scan -- the prefill of hs_linattn_prefill_from_state for calls
+ * with few problems: the segments of each problem's tail run in parallel.
+ *
+ * Paper: as hs_linattn_prefill_from_state (Section 2.2, Section 4.1 and Table 2).
+ * The recurrence is linear in the state, so over a segment [s,e) of the absolute
+ * 64-token grid S_e = diag(G) S_s + dS with G = exp(sum of the segment's log-gates)
+ * and dS the segment's state from the zero state.  Three launches: the tensor-core
+ * kernel runs every segment as a problem of its own from the zero state (dS), an
+ * elementwise scan chains S_{n+1} = G_n S_n + dS_n per (problem, head) and writes
+ * the checkpoints and the final state, and the tensor-core kernel runs every
+ * segment again from its start state S_n for the outputs.  A call with one problem
+ * of 16 heads then occupies (segments x 16) CTAs instead of 16.
+ *
+ * Results: the outputs, final states and checkpoints of the same recurrence, within
+ * the same accuracy as hs_linattn_prefill_from_state (the two are not bit-identical:
+ * here the state enters each segment through the scan's fma instead of the tensor-
+ * core accumulation).  Every step depends only on the segment's inputs and the state
+ * it starts from, so resuming at a multiple of HS_CHUNK with this call reproduces a
+ * full recomputation with this call bit for bit.
+ *
+ * Arguments as hs_linattn_prefill_from_state (shp->kernel AUTO or CHUNKED_TC: the
+ * segments run on the tensor-core kernel), plus
+ *   workspace        device memory the call uses between its launches, 16-byte
+ *                    aligned, at least hs_linattn_scan_workspace_bytes bytes: two float
+ *                    states per segment (2 x segments x n_heads x d_k x d_v x 4 bytes);
+ *                    its contents on entry are ignored and on return undefined
+ *   workspace_bytes  its size
+ * The rows t >= n_tokens[b] of o are not written.  The workspace must not overlap
+ * any other argument, and concurrent calls need their own workspaces.
+ * Errors: as hs_linattn_prefill_from_state; HS_ERR_INVALID_ARG also for a NULL or
+ * too small workspace, HS_ERR_MISALIGNED for a misaligned one, HS_ERR_UNSUPPORTED
+ * for another kernel choice.
+ */
+hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q,
+                                  const uint16_t *k, const uint16_t *v, const float *log_g,
+                                  float *o, float *state, const int64_t *pos0,
+                                  const int32_t *n_tokens, int32_t ckpt_interval,
+                                  float *const *ckpt_slots, void *workspace,
+                                  int64_t workspace_bytes, int32_t *d_err, cudaStream_t stream);
+
+/*
+ * hs_linattn_scan_workspace_bytes -- the workspace hs_linattn_prefill_scan needs for
+ * these arguments (host only): 2 x segments x n_heads x d_k x d_v x 4 bytes, with
+ * segments = sum over b of ceil((pos0[b] + n_tokens[b]) / 64) - floor(pos0[b] / 64)
+ * for n_tokens[b] > 0.  Errors: the shape and argument checks of the call.
+ */
+hs_status hs_linattn_scan_workspace_bytes(const hs_linattn_shape *shp, const int64_t *pos0,
+                                          const int32_t *n_tokens, int64_t *bytes_out);
+
+/*
  * hs_linattn_num_checkpoints -- number of checkpoint slots the prefill above
  * writes for these arguments (host only): the sum over b of
  * floor((pos0[b]+n_tokens[b])/C) - floor(pos0[b]/C), 0 when C == 0.

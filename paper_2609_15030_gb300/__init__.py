@@ -44,7 +44,7 @@ EXPORTED = ("hs_status_string", "hs_version", "hs_align_prefix", "hs_restore_kv_
             "hs_save_kv_pages", "hs_restore_kv_page_slices", "hs_save_kv_page_slices",
             "hs_restore_state", "hs_checkpoint_states", "hs_linattn_prefill_from_state",
             "hs_linattn_num_checkpoints", "hs_linattn_prefill_packed", "hs_restore_request",
-            "hs_test_prefill_stalled")
+            "hs_test_prefill_stalled", "hs_linattn_prefill_scan", "hs_linattn_scan_workspace_bytes")
 
 
 class HsError(RuntimeError):
@@ -91,6 +91,9 @@ def load() -> C.CDLL:
             L.hs_linattn_prefill_packed.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp, vp,
                                                     vp, vp, vp, vp, vp, i32, vp, vp, vp]
             L.hs_test_prefill_stalled.argtypes = L.hs_linattn_prefill_from_state.argtypes
+            L.hs_linattn_prefill_scan.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp, vp, vp,
+                                                  vp, vp, vp, i32, vp, vp, i64, vp, vp]
+            L.hs_linattn_scan_workspace_bytes.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp]
             for name in EXPORTED[2:]:
                 getattr(L, name).restype = C.c_int
             _lib = L
@@ -237,6 +240,33 @@ def hs_test_prefill_stalled(shape: hs_linattn_shape, q, k, v, log_g, o, state, p
     nothing completes; each CTA's bounded wait runs out and it reports HS_DEVERR_TIMEOUT."""
     _prefill_call("hs_test_prefill_stalled", shape, q, k, v, log_g, o, state, pos0, n_tokens,
                   ckpt_interval, ckpt_slots, d_err, stream)
+
+
+def hs_linattn_scan_workspace_bytes(shape: hs_linattn_shape, pos0, n_tokens) -> int:
+    """Bytes of workspace hs_linattn_prefill_scan needs for these arguments."""
+    B = int(shape.batch)
+    p0 = (C.c_int64 * max(B, 1))(*[int(x) for x in pos0])
+    nt = (C.c_int32 * max(B, 1))(*[int(x) for x in n_tokens])
+    out = C.c_int64()
+    rc = load().hs_linattn_scan_workspace_bytes(C.byref(shape), C.addressof(p0), C.addressof(nt),
+                                                C.addressof(out))
+    _check(rc, "hs_linattn_scan_workspace_bytes")
+    return out.value
+
+
+def hs_linattn_prefill_scan(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0, n_tokens,
+                            ckpt_interval: int, ckpt_slots, workspace, workspace_bytes: int,
+                            d_err=None, stream=None):
+    """Segment-parallel prefill (same arguments as hs_linattn_prefill_from_state plus a device
+    workspace of hs_linattn_scan_workspace_bytes bytes)."""
+    B = int(shape.batch)
+    p0 = (C.c_int64 * max(B, 1))(*[int(x) for x in pos0])
+    nt = (C.c_int32 * max(B, 1))(*[int(x) for x in n_tokens])
+    rc = load().hs_linattn_prefill_scan(C.byref(shape), _ptr(q), _ptr(k), _ptr(v), _ptr(log_g),
+                                        _ptr(o), _ptr(state), C.addressof(p0), C.addressof(nt),
+                                        int(ckpt_interval), _ptr(ckpt_slots), _ptr(workspace),
+                                        int(workspace_bytes), _ptr(d_err), _stream(stream))
+    _check(rc, "hs_linattn_prefill_scan")
 
 
 def hs_linattn_prefill_packed(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0, n_tokens,

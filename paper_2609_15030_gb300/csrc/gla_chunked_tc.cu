@@ -228,11 +228,16 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // largest magnitude.  The builders meanwhile stage and build the first segment.
     float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
     if (worker) {
-        state_load<D>(smem, tmem, st_g);
+        state_load<D>(smem, tmem, p.zero_state ? nullptr : st_g);
         tc_fence_before();
         bar_staters();
         tc_fence_after();
     }
+
+    // the output rows from local token t (nullptr: this launch writes no outputs)
+    auto outp = [&](int64_t t) -> float * {
+        return p.o != nullptr ? p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D : nullptr;
+    };
 
     // ---- a short segment (<= kShort tokens, staged inputs already waited for, no decay
     // pending): the per-token recurrence with the recurrent kernel's exact operation order
@@ -241,7 +246,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         short_state<D>(smem, tmem, L, ckpt_slot(seg_end));
         if (tid == kLoader && seg_end < end)
             issue_tma(tok_s + L);
-        short_outputs<D>(smem, L, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride);
+        short_outputs<D>(smem, L, outp(tok_s), tstride);
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -302,7 +307,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (!wait_all(kIssuer, bar_s, ph_s))
             return false;
         state_pass<D>(smem, tmem, -1, ckpt_slot(seg_end), false);   // checkpoint and |S| of the final state
-        out_epilogue<D>(tmem, p.o + (((int64_t)p.row0[b] + tok_s) * p.n_heads + h) * D, tstride, L, par, false);
+        out_epilogue<D>(tmem, outp(tok_s), tstride, L, par, false);
         tc_fence_before();
         __syncthreads();
         tc_fence_after();
@@ -322,7 +327,6 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // such a segment starts a new run, whose first decision reads the measured state exactly as
     // a run resumed from a checkpoint at that segment does.  The groups then meet CTA-wide.
     // No MMA is in flight at either end.
-    auto outp = [&](int64_t t) { return p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D; };
     int kseq = 0;   // long segments of the current run so far (slot of 2^{Lam_last}: kseq mod 4)
     auto builder_run = [&](int64_t rpos, int64_t rtok) {
         int par = 0;
@@ -525,7 +529,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     }
 
     if (!aborted) {
-        state_store<D>(tmem, st_g);   // final state back to global memory, row = key dim
+        if (!p.no_state_out)
+            state_store<D>(tmem, st_g);   // final state back to global memory, row = key dim
     } else {
         // let this CTA's own copies and MMAs drain (bounded) before its memory goes away
         if (tid == kLoader) {

@@ -1,6 +1,7 @@
 // C-ABI entry points of libhs: host-side validation, then one launch per call.
 // Validation happens before any CUDA runtime call, so argument errors are
 // reported without touching the GPU.
+#include <algorithm>
 #include <cstring>
 
 #include "hs_internal.cuh"
@@ -384,6 +385,175 @@ hs_status hs_test_prefill_stalled(const hs_linattn_shape *shp, const uint16_t *q
 {
     return prefill(shp, q, k, v, log_g, o, state, pos0, n_tokens, nullptr, ckpt_interval,
                    ckpt_slots, d_err, stream, true);
+}
+
+// ---- the segment-parallel prefill: every segment from the zero state, a state scan, every
+// segment from its start state ----
+
+// segments of [pos0, pos0 + n) on the HS_CHUNK grid
+static int64_t n_segments(int64_t pos0, int64_t n)
+{
+    return n > 0 ? (pos0 + n + HS_CHUNK - 1) / HS_CHUNK - pos0 / HS_CHUNK : 0;
+}
+
+// the checks of hs_linattn_prefill_from_state that do not touch device memory, and the
+// number of segments; HS_OK with *n_seg = 0 when there is nothing to compute
+static hs_status scan_check(const hs_linattn_shape *shp, const int64_t *pos0,
+                            const int32_t *n_tokens, int64_t *n_seg)
+{
+    if (shp == nullptr || n_seg == nullptr)
+        return HS_ERR_INVALID_ARG;
+    const hs_linattn_shape s = *shp;
+    if (s.batch < 0 || s.n_heads < 1 || s.max_tokens < 0 || s.reserved != 0)
+        return HS_ERR_INVALID_ARG;
+    if (s.kernel != HS_LINATTN_AUTO && s.kernel != HS_LINATTN_CHUNKED_TC)
+        return s.kernel >= HS_LINATTN_AUTO && s.kernel <= HS_LINATTN_SINGLE_TOKEN
+                   ? HS_ERR_UNSUPPORTED : HS_ERR_INVALID_ARG;
+    if (s.d_k != s.d_v || (s.d_k != 64 && s.d_k != 128))
+        return HS_ERR_UNSUPPORTED;
+    if (s.batch > HS_MAX_BATCH)
+        return HS_ERR_UNSUPPORTED;
+    *n_seg = 0;
+    if (s.batch > 0 && (pos0 == nullptr || n_tokens == nullptr))
+        return HS_ERR_INVALID_ARG;
+    int64_t total = 0;
+    for (int32_t b = 0; b < s.batch; ++b) {
+        if (pos0[b] < 0 || n_tokens[b] < 0 || pos0[b] > ((int64_t)1 << 40) ||
+            (int64_t)n_tokens[b] > s.max_tokens)
+            return HS_ERR_INVALID_ARG;
+        if ((int64_t)b * s.max_tokens + n_tokens[b] > INT32_MAX)
+            return HS_ERR_UNSUPPORTED;   // token rows are 32-bit
+        total += n_segments(pos0[b], n_tokens[b]);
+    }
+    if (total > INT32_MAX)
+        return HS_ERR_UNSUPPORTED;
+    *n_seg = total;
+    return HS_OK;
+}
+
+hs_status hs_linattn_scan_workspace_bytes(const hs_linattn_shape *shp, const int64_t *pos0,
+                                          const int32_t *n_tokens, int64_t *bytes_out)
+{
+    if (bytes_out == nullptr)
+        return HS_ERR_INVALID_ARG;
+    int64_t n_seg = 0;
+    const hs_status st = scan_check(shp, pos0, n_tokens, &n_seg);
+    if (st != HS_OK)
+        return st;
+    *bytes_out = 2 * n_seg * shp->n_heads * (int64_t)shp->d_k * shp->d_v * 4;
+    return HS_OK;
+}
+
+hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q,
+                                  const uint16_t *k, const uint16_t *v, const float *log_g,
+                                  float *o, float *state, const int64_t *pos0,
+                                  const int32_t *n_tokens, int32_t ckpt_interval,
+                                  float *const *ckpt_slots, void *workspace,
+                                  int64_t workspace_bytes, int32_t *d_err, cudaStream_t stream)
+{
+    int64_t n_seg = 0;
+    hs_status st = scan_check(shp, pos0, n_tokens, &n_seg);
+    if (st != HS_OK)
+        return st;
+    const hs_linattn_shape s = *shp;
+    if (ckpt_interval < 0)
+        return HS_ERR_INVALID_ARG;
+    if (ckpt_interval % HS_CHUNK != 0)
+        return HS_ERR_UNSUPPORTED;
+    if (n_seg == 0)
+        return HS_OK;
+    if (q == nullptr || k == nullptr || v == nullptr || log_g == nullptr || o == nullptr ||
+        state == nullptr || workspace == nullptr)
+        return HS_ERR_INVALID_ARG;
+    if (misaligned16(q) || misaligned16(k) || misaligned16(v) || misaligned16(log_g) ||
+        misaligned16(o) || misaligned16(state) || misaligned16(workspace))
+        return HS_ERR_MISALIGNED;
+    const int64_t D = s.d_k;
+    const int64_t per = (int64_t)s.n_heads * D * D;     // floats of one segment's state
+    if (workspace_bytes < 2 * n_seg * per * 4)
+        return HS_ERR_INVALID_ARG;
+    float *ws_dS = static_cast<float *>(workspace);
+    float *ws_Sn = ws_dS + n_seg * per;
+
+    // the scan's parameters (the original problems) and the segments' first rows
+    hs::ScanParams sp;
+    std::memset(&sp, 0, sizeof sp);
+    sp.log_g = log_g;
+    sp.state = state;
+    sp.dS = ws_dS;
+    sp.Sn = ws_Sn;
+    sp.ckpt_slots = (ckpt_interval > 0) ? ckpt_slots : nullptr;
+    sp.d_err = d_err;
+    sp.batch = s.batch;
+    sp.n_heads = s.n_heads;
+    sp.ckpt_interval = (sp.ckpt_slots != nullptr) ? ckpt_interval : 0;
+    int64_t seg = 0, ck = 0;
+    for (int32_t b = 0; b < s.batch; ++b) {
+        sp.pos0[b] = pos0[b];
+        sp.n_tokens[b] = n_tokens[b];
+        sp.row0[b] = (int32_t)((int64_t)b * s.max_tokens);
+        sp.ck_base[b] = (int32_t)ck;
+        sp.seg_base[b] = (int32_t)seg;
+        seg += n_segments(pos0[b], n_tokens[b]);
+        if (sp.ckpt_interval > 0 && n_tokens[b] > 0)
+            ck += (pos0[b] + n_tokens[b]) / sp.ckpt_interval - pos0[b] / sp.ckpt_interval;
+    }
+    if (ck > INT32_MAX)
+        return HS_ERR_INVALID_ARG;
+
+    // one tensor-core pass over every segment as a problem of its own, at most HS_MAX_BATCH
+    // segments per launch: from the zero state, writing each segment's state into dS and no
+    // outputs; or from the scanned start states Sn, writing the outputs and no states
+    auto pass = [&](bool from_zero) -> hs_status {
+        hs::GlaParams p;
+        int32_t j = 0;
+        int64_t first = 0;
+        auto flush = [&]() -> hs_status {
+            if (j == 0)
+                return HS_OK;
+            p.batch = j;
+            p.state = (from_zero ? ws_dS : ws_Sn) + first * per;
+            const hs_status r = cuda_status(hs::launch_gla_chunked_tc(p, (int)D, stream));
+            first += j;
+            j = 0;
+            return r;
+        };
+        auto reset = [&]() {
+            std::memset(&p, 0, sizeof p);
+            p.q = q;
+            p.k = k;
+            p.v = v;
+            p.log_g = log_g;
+            p.o = from_zero ? nullptr : o;
+            p.d_err = d_err;
+            p.n_heads = s.n_heads;
+            p.zero_state = from_zero ? 1 : 0;
+            p.no_state_out = from_zero ? 0 : 1;
+        };
+        reset();
+        for (int32_t b = 0; b < s.batch; ++b) {
+            const int64_t end = pos0[b] + n_tokens[b];
+            for (int64_t at = pos0[b]; at < end;) {
+                const int64_t e = std::min<int64_t>(end, (at / HS_CHUNK + 1) * HS_CHUNK);
+                p.pos0[j] = at;
+                p.n_tokens[j] = (int32_t)(e - at);
+                p.row0[j] = (int32_t)((int64_t)b * s.max_tokens + (at - pos0[b]));
+                at = e;
+                if (++j == HS_MAX_BATCH) {
+                    const hs_status r = flush();
+                    if (r != HS_OK)
+                        return r;
+                    reset();
+                }
+            }
+        }
+        return flush();
+    };
+    if ((st = pass(true)) != HS_OK)
+        return st;
+    if ((st = cuda_status(hs::launch_gla_scan(sp, (int)D, stream))) != HS_OK)
+        return st;
+    return pass(false);
 }
 
 hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t *q,

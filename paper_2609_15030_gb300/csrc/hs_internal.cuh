@@ -70,6 +70,10 @@ struct GlaParams {
     int32_t n_heads;
     int32_t ckpt_interval;     // 0: none
     int32_t stall_for_test;    // tensor-core kernel only: one wait that nothing completes (failure-detection tests)
+    int32_t zero_state;        // tensor-core kernel only: start every problem from the zero state
+                               // (state is then only written)
+    int32_t no_state_out;      // tensor-core kernel only: the final state is not written
+                               // (o == nullptr: no outputs are written either)
     int64_t pos0[HS_MAX_BATCH];
     int32_t n_tokens[HS_MAX_BATCH];
     int32_t ck_base[HS_MAX_BATCH];  // index of the problem's first slot in ckpt_slots
@@ -94,6 +98,27 @@ cudaError_t launch_restore_request(const void *const *staging, void *const *cach
                                    int32_t *d_err, int sm_count, cudaStream_t s);
 cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t n,
                              int64_t floats_each, int32_t *d_err, int sm_count, cudaStream_t s);
+// The elementwise state scan between the two tensor-core passes of hs_linattn_prefill_scan:
+// per (problem, head), S_{n+1} = g_n * S_n + dS_n over the problem's segments (g_n the
+// segment's decay factor per key dim, dS_n the segment's state from the zero state), recording
+// each segment's start state, the checkpoints and the final state.
+struct ScanParams {
+    const float *log_g;       // [rows][n_heads][d]
+    float *state;             // [batch][n_heads][d][d]: in the state at pos0, out at pos0 + n
+    const float *dS;          // [segments][n_heads][d][d]: each segment from the zero state
+    float *Sn;                // [segments][n_heads][d][d]: each segment's start state (written)
+    float *const *ckpt_slots; // as GlaParams
+    int32_t *d_err;
+    int32_t batch;
+    int32_t n_heads;
+    int32_t ckpt_interval;
+    int64_t pos0[HS_MAX_BATCH];
+    int32_t n_tokens[HS_MAX_BATCH];
+    int32_t row0[HS_MAX_BATCH];
+    int32_t ck_base[HS_MAX_BATCH];
+    int32_t seg_base[HS_MAX_BATCH];   // index of the problem's first segment in dS / Sn
+};
+cudaError_t launch_gla_scan(const ScanParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_decode(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s);

@@ -266,6 +266,41 @@ def test_packed_prefill_host_validation():
     call(n_tokens=[0, 0], q=None, k=None, v=None, log_g=None, o=None)   # empty tails: OK
 
 
+def test_scan_prefill_host_validation():
+    """hs_linattn_prefill_scan: the prefill's argument checks plus its workspace, and the
+    workspace size it asks for, all on the host before any CUDA call."""
+    sh = hs.make_shape(2, 4, 128, 128, 200)
+    # two states per segment: problem 0 spans [100, 300) -> 4 segments, problem 1 [0, 64) -> 1
+    assert hs.hs_linattn_scan_workspace_bytes(sh, [100, 0], [200, 64]) == 2 * 5 * 4 * 128 * 128 * 4
+    assert hs.hs_linattn_scan_workspace_bytes(sh, [0, 0], [0, 0]) == 0
+    need = 2 * 5 * 4 * 128 * 128 * 4
+
+    def call(shape=sh, **kw):
+        a = dict(q=FAKE, k=FAKE, v=FAKE, log_g=FAKE, o=FAKE, state=FAKE, pos0=[100, 0],
+                 n_tokens=[200, 64], ckpt_interval=64, ckpt_slots=None, workspace=FAKE,
+                 workspace_bytes=need, d_err=None, stream=0)
+        a.update(kw)
+        hs.hs_linattn_prefill_scan(shape, **a)
+    cases = [
+        (dict(workspace=None), hs.HS_ERR_INVALID_ARG),
+        (dict(workspace_bytes=need - 16), hs.HS_ERR_INVALID_ARG),
+        (dict(workspace=FAKE + 8), hs.HS_ERR_MISALIGNED),
+        (dict(shape=hs.make_shape(2, 4, 128, 128, 200, hs.HS_LINATTN_RECURRENT)),
+         hs.HS_ERR_UNSUPPORTED),
+        (dict(shape=hs.make_shape(2, 4, 96, 96, 200)), hs.HS_ERR_UNSUPPORTED),
+        (dict(n_tokens=[201, 64]), hs.HS_ERR_INVALID_ARG),
+        (dict(pos0=[-1, 0]), hs.HS_ERR_INVALID_ARG),
+        (dict(ckpt_interval=96), hs.HS_ERR_UNSUPPORTED),
+        (dict(state=None), hs.HS_ERR_INVALID_ARG),
+        (dict(o=FAKE + 4), hs.HS_ERR_MISALIGNED),
+    ]
+    for kw, code in cases:
+        with pytest.raises(hs.HsError) as e:
+            call(**kw)
+        assert e.value.status == code, kw
+    call(n_tokens=[0, 0], q=None, workspace=None, workspace_bytes=0)   # nothing to compute: OK
+
+
 def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     import importlib
     mod = importlib.import_module("paper_2609_15030_gb300")
