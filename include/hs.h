@@ -52,7 +52,9 @@ typedef enum hs_status {
     HS_ERR_MISALIGNED = 2,    /* pointer or byte size not a multiple of 16 bytes */
     HS_ERR_UNSUPPORTED = 3,   /* shape outside what the kernels implement (see each call) */
     HS_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed */
-    HS_ERR_DEVICE_CHECK = 5   /* reserved for callers that fold d_err into a status */
+    HS_ERR_DEVICE_CHECK = 5,  /* reserved for callers that fold d_err into a status */
+    HS_ERR_TOO_LARGE = 6      /* the call needs more than the library's fixed workspace
+                                 (HS_NOALLOC_SCRATCH_BYTES) holds */
 } hs_status;
 
 /* codes a kernel may store into d_err */
@@ -418,6 +420,43 @@ hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q
  */
 hs_status hs_linattn_scan_workspace_bytes(const hs_linattn_shape *shp, const int64_t *pos0,
                                           const int32_t *n_tokens, int64_t *bytes_out);
+
+/* Size of the fixed device workspace of hs_linattn_prefill_scan_noalloc (16 MiB per device):
+ * room for 2 x 8 segments x 16 heads x 128 x 128 floats, e.g. one 512-token tail of 16
+ * heads at d = 128 that starts on the 64-token grid. */
+#define HS_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/*
+ * hs_linattn_prefill_scan_noalloc -- hs_linattn_prefill_scan for callers that cannot
+ * allocate device memory when they resume a request.
+ *
+ * The paper has no counterpart: it is a calling convention of this library.  Some callers
+ * have no device memory to give out at that point: a serving engine commonly reserves
+ * nearly all free HBM for its KV-cache block pool at start-up and allocates only from its
+ * own pools afterwards, and its scheduler loop cannot take the device-wide synchronisation
+ * that cudaMalloc or cudaFree may cause.  This call takes the workspace from a fixed array
+ * of HS_NOALLOC_SCRATCH_BYTES bytes that the library keeps on each device, and calls no
+ * allocating routine.
+ *
+ * Arguments, results and errors: as hs_linattn_prefill_scan without workspace and
+ * workspace_bytes, plus HS_ERR_TOO_LARGE when hs_linattn_scan_workspace_bytes for these
+ * arguments exceeds HS_NOALLOC_SCRATCH_BYTES (checked on the host before any CUDA call), and
+ * HS_ERR_CUDA when the set-up below fails.
+ * Set-up: the first call on a device that has tokens to compute looks up the array's
+ * address there (cudaGetSymbolAddress, with the current device, which loads the array if
+ * the library's module is loaded lazily) and caches it; make that first call before any
+ * stream capture.  The stream must belong to the current device.
+ * Sharing: every call on a device uses the same array and finds the previous call's data
+ * in it; nothing has to be cleared, since a call writes every word it reads first.  Calls
+ * that can run at the same time on the GPU (two streams, or host threads without an order
+ * between their calls) corrupt each other's workspace: serialise them.
+ */
+hs_status hs_linattn_prefill_scan_noalloc(const hs_linattn_shape *shp, const uint16_t *q,
+                                          const uint16_t *k, const uint16_t *v,
+                                          const float *log_g, float *o, float *state,
+                                          const int64_t *pos0, const int32_t *n_tokens,
+                                          int32_t ckpt_interval, float *const *ckpt_slots,
+                                          int32_t *d_err, cudaStream_t stream);
 
 /*
  * hs_linattn_num_checkpoints -- number of checkpoint slots the prefill above

@@ -24,6 +24,7 @@ HS_ERR_MISALIGNED = 2
 HS_ERR_UNSUPPORTED = 3
 HS_ERR_CUDA = 4
 HS_ERR_DEVICE_CHECK = 5
+HS_ERR_TOO_LARGE = 6
 
 HS_DEVERR_NONE = 0
 HS_DEVERR_BLOCK_OOB = 1
@@ -34,6 +35,7 @@ HS_DEVERR_TIMEOUT = 4
 HS_MAX_BATCH = 384
 HS_CHUNK = 64
 HS_SHORT_SEGMENT = 8
+HS_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 HS_LINATTN_AUTO = 0
 HS_LINATTN_RECURRENT = 1
@@ -44,7 +46,8 @@ EXPORTED = ("hs_status_string", "hs_version", "hs_align_prefix", "hs_restore_kv_
             "hs_save_kv_pages", "hs_restore_kv_page_slices", "hs_save_kv_page_slices",
             "hs_restore_state", "hs_checkpoint_states", "hs_linattn_prefill_from_state",
             "hs_linattn_num_checkpoints", "hs_linattn_prefill_packed", "hs_restore_request",
-            "hs_test_prefill_stalled", "hs_linattn_prefill_scan", "hs_linattn_scan_workspace_bytes")
+            "hs_test_prefill_stalled", "hs_linattn_prefill_scan", "hs_linattn_scan_workspace_bytes",
+            "hs_linattn_prefill_scan_noalloc")
 
 
 class HsError(RuntimeError):
@@ -94,6 +97,8 @@ def load() -> C.CDLL:
             L.hs_linattn_prefill_scan.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp, vp, vp,
                                                   vp, vp, vp, i32, vp, vp, i64, vp, vp]
             L.hs_linattn_scan_workspace_bytes.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp]
+            L.hs_linattn_prefill_scan_noalloc.argtypes = [C.POINTER(hs_linattn_shape), vp, vp, vp,
+                                                          vp, vp, vp, vp, vp, i32, vp, vp, vp]
             for name in EXPORTED[2:]:
                 getattr(L, name).restype = C.c_int
             _lib = L
@@ -267,6 +272,26 @@ def hs_linattn_prefill_scan(shape: hs_linattn_shape, q, k, v, log_g, o, state, p
                                         int(ckpt_interval), _ptr(ckpt_slots), _ptr(workspace),
                                         int(workspace_bytes), _ptr(d_err), _stream(stream))
     _check(rc, "hs_linattn_prefill_scan")
+
+
+def hs_linattn_prefill_scan_noalloc(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0,
+                                    n_tokens, ckpt_interval: int, ckpt_slots=None, d_err=None,
+                                    stream=None):
+    """hs_linattn_prefill_scan with the library's fixed per-device workspace of
+    HS_NOALLOC_SCRATCH_BYTES, for callers that cannot allocate device memory at this point (a
+    serving engine whose HBM is already handed to its KV-cache pool).  Allocates nothing: the
+    host arrays below are ctypes buffers.  Calls that overlap on the GPU share the workspace
+    and race; the first call on a device does a one-time set-up and belongs before any stream
+    capture."""
+    B = int(shape.batch)
+    p0 = (C.c_int64 * max(B, 1))(*[int(x) for x in pos0])
+    nt = (C.c_int32 * max(B, 1))(*[int(x) for x in n_tokens])
+    rc = load().hs_linattn_prefill_scan_noalloc(C.byref(shape), _ptr(q), _ptr(k), _ptr(v),
+                                                _ptr(log_g), _ptr(o), _ptr(state),
+                                                C.addressof(p0), C.addressof(nt),
+                                                int(ckpt_interval), _ptr(ckpt_slots),
+                                                _ptr(d_err), _stream(stream))
+    _check(rc, "hs_linattn_prefill_scan_noalloc")
 
 
 def hs_linattn_prefill_packed(shape: hs_linattn_shape, q, k, v, log_g, o, state, pos0, n_tokens,

@@ -58,6 +58,8 @@ const char *hs_status_string(hs_status s)
     case HS_ERR_UNSUPPORTED: return "HS_ERR_UNSUPPORTED: shape not implemented";
     case HS_ERR_CUDA: return "HS_ERR_CUDA: CUDA runtime call or launch failed";
     case HS_ERR_DEVICE_CHECK: return "HS_ERR_DEVICE_CHECK: a kernel reported an error";
+    case HS_ERR_TOO_LARGE:
+        return "HS_ERR_TOO_LARGE: the call needs more than the library's fixed workspace";
     }
     return "unknown hs_status";
 }

@@ -43,7 +43,7 @@ def test_exports_every_declared_symbol():
 
 
 def test_status_strings_and_version():
-    for s in range(6):
+    for s in range(7):
         assert hs.hs_status_string(s).startswith("HS_")
     assert "unknown" in hs.hs_status_string(99)
     assert hs.hs_version() >= 100
@@ -299,6 +299,42 @@ def test_scan_prefill_host_validation():
             call(**kw)
         assert e.value.status == code, kw
     call(n_tokens=[0, 0], q=None, workspace=None, workspace_bytes=0)   # nothing to compute: OK
+
+
+def test_noalloc_scan_rejects_on_the_host():
+    """hs_linattn_prefill_scan_noalloc: calls whose workspace would exceed the fixed 16 MiB
+    are refused with HS_ERR_TOO_LARGE, and argument errors are reported, before any CUDA call
+    (this host has no GPU, so a call that reached the CUDA runtime would fail otherwise)."""
+    assert hs.HS_NOALLOC_SCRATCH_BYTES == 16 << 20
+    sh = hs.make_shape(1, 16, 128, 128, 1024)
+    # 512 tokens from 4096: 8 segments x 16 heads x 2 states of 64 KiB = exactly the limit
+    assert hs.hs_linattn_scan_workspace_bytes(sh, [4096], [512]) == hs.HS_NOALLOC_SCRATCH_BYTES
+
+    def call(shape=sh, **kw):
+        a = dict(q=FAKE, k=FAKE, v=FAKE, log_g=FAKE, o=FAKE, state=FAKE, pos0=[4096],
+                 n_tokens=[512], ckpt_interval=512, ckpt_slots=None, d_err=None, stream=0)
+        a.update(kw)
+        hs.hs_linattn_prefill_scan_noalloc(shape, **a)
+    cases = [
+        (dict(n_tokens=[513]), hs.HS_ERR_TOO_LARGE),            # one more segment
+        (dict(pos0=[4095]), hs.HS_ERR_TOO_LARGE),               # off the grid: 9 segments
+        (dict(shape=hs.make_shape(2, 16, 128, 128, 1024), pos0=[0, 0], n_tokens=[256, 320]),
+         hs.HS_ERR_TOO_LARGE),
+        (dict(shape=hs.make_shape(1, 16, 128, 128, 1024, hs.HS_LINATTN_RECURRENT)),
+         hs.HS_ERR_UNSUPPORTED),
+        (dict(n_tokens=[1025]), hs.HS_ERR_INVALID_ARG),
+        (dict(ckpt_interval=-64), hs.HS_ERR_INVALID_ARG),
+        (dict(ckpt_interval=96), hs.HS_ERR_UNSUPPORTED),
+        (dict(q=None), hs.HS_ERR_INVALID_ARG),
+        (dict(state=None, o=FAKE + 4), hs.HS_ERR_INVALID_ARG),
+        (dict(o=FAKE + 4), hs.HS_ERR_MISALIGNED),
+    ]
+    for kw, code in cases:
+        with pytest.raises(hs.HsError) as e:
+            call(**kw)
+        assert e.value.status == code, kw
+    assert "fixed workspace" in hs.hs_status_string(hs.HS_ERR_TOO_LARGE)
+    call(n_tokens=[0], q=None, state=None)      # nothing to compute: OK, no set-up
 
 
 def test_missing_library_fails_loudly(monkeypatch, tmp_path):
