@@ -88,7 +88,8 @@ KERNEL_OF = {"decode": "gla_decode_kernel<128>", "prefill": "gla_chunked_tc_kern
 KERNEL_SRC = {"gla_decode_kernel": "gla_decode.cu", "gla_chunked_tc_kernel": "gla_chunked_tc.cu",
               "gla_recurrent_kernel": "gla_recurrent.cu", "restore_request_kernel": "restore_request.cu",
               "kv_scatter_kernel": "kv_scatter.cu", "kv_gather_kernel": "kv_scatter.cu",
-              "kv_slices_kernel": "kv_scatter.cu", "slot_copy_kernel": "slot_copy.cu"}
+              "kv_slices_kernel": "kv_scatter.cu", "slot_copy_kernel": "slot_copy.cu",
+              "gla_scan_kernel": "gla_scan.cu"}
 DTYPE = "bf16 q/k/v, fp32 log-gates; fp16 (fast) or tf32 (exact) MMA operands, fp32 accumulate, state and outputs"
 
 
@@ -914,13 +915,13 @@ def _l2_flush(torch, dev, buf=[]):
     buf[0].fill_(1)
 
 
-def sweep_run(dev, reps=10, scan=True):
+def sweep_run(dev, reps=10, scan=True, seq=True, lengths=None):
     """Single-layer kernel sweep: one linear layer, 16 heads, d = 128, checkpoints every 512,
     batch 1.  For each L in 512..4608: the resumed tail prefill (c = C floor((L-1)/C), 512
     tokens from the state at c, emitting the checkpoint at L; the hit L-37 aligns to the same
     c) and the recomputation of [0,L) from the zero state emitting every checkpoint; with
-    `scan`, both also through the segment-parallel prefill.  Each call is timed alone between
-    CUDA events with L2 flushed before it; median of `reps`."""
+    `scan`, both also through the segment-parallel prefill (`seq=False`: only there).  Each
+    call is timed alone between CUDA events with L2 flushed before it; median of `reps`."""
     import torch
     import paper_2609_15030_gb300 as hs
     from hs_inputs import SWEEP, torch_gen_linear
@@ -940,7 +941,7 @@ def sweep_run(dev, reps=10, scan=True):
     ws_bytes = hs.hs_linattn_scan_workspace_bytes(shape, [0], [Lmax])
     ws = torch.empty((ws_bytes // 4,), device=dev)
     rows = []
-    for L in SWEEP_LENGTHS:
+    for L in (lengths or SWEEP_LENGTHS):
         c, _, tail = hs.hs_align_prefix(L, L, list(range(C, L + 1, C)), S.page)
         c37, _, _ = hs.hs_align_prefix(L, L - 37, list(range(C, L + 1, C)), S.page)
         nck_t = hs.hs_linattn_num_checkpoints([c], [tail], C)
@@ -969,7 +970,7 @@ def sweep_run(dev, reps=10, scan=True):
                                        ws_bytes, None, stream.cuda_stream)
         res = {}
         arms = [("tail", resume, lambda: state.copy_(ck)),
-                ("recompute", recompute, lambda: state.zero_())]
+                ("recompute", recompute, lambda: state.zero_())] if seq else []
         if scan:
             arms += [("tail_scan", resume_scan, lambda: state.copy_(ck)),
                      ("recompute_scan", recompute_scan, lambda: state.zero_())]
@@ -991,16 +992,17 @@ def sweep_run(dev, reps=10, scan=True):
         b_rec = gla_bytes(1, nH, d, L, L // C)
         tp_t = tensor.get(f"gla_chunked_tc_kernel@sweep_tail_{L}")
         tp_r = tensor.get(f"gla_chunked_tc_kernel@sweep_recompute_{L}")
-        rows.append({
-            "L": L, "c": c, "c_hit_L-37": c37, "tail": tail,
-            "tail_us": round(res["tail"] * 1e6, 2),
-            "tail_tokens_per_s": round(tail / res["tail"], 1),
-            "tail_hbm_frac": round(b_tail / res["tail"] / 1e9 / peak, 4),
-            "tail_tensor_pipe": tp_t["active"] if tp_t else None,
-            "recompute_us": round(res["recompute"] * 1e6, 2),
-            "recompute_tokens_per_s": round(L / res["recompute"], 1),
-            "recompute_hbm_frac": round(b_rec / res["recompute"] / 1e9 / peak, 4),
-            "recompute_tensor_pipe": tp_r["active"] if tp_r else None})
+        rows.append({"L": L, "c": c, "c_hit_L-37": c37, "tail": tail})
+        if seq:
+            rows[-1].update({
+                "tail_us": round(res["tail"] * 1e6, 2),
+                "tail_tokens_per_s": round(tail / res["tail"], 1),
+                "tail_hbm_frac": round(b_tail / res["tail"] / 1e9 / peak, 4),
+                "tail_tensor_pipe": tp_t["active"] if tp_t else None,
+                "recompute_us": round(res["recompute"] * 1e6, 2),
+                "recompute_tokens_per_s": round(L / res["recompute"], 1),
+                "recompute_hbm_frac": round(b_rec / res["recompute"] / 1e9 / peak, 4),
+                "recompute_tensor_pipe": tp_r["active"] if tp_r else None})
         if scan:
             rows[-1].update({
                 "tail_scan_us": round(res["tail_scan"] * 1e6, 2),
@@ -1423,6 +1425,13 @@ def run_case(name: str, iters: int = 5):
         r = sweep_run(dev, reps=1, scan=False)
         for row in r["rows"]:
             print(json.dumps({k: row[k] for k in ("L", "tail_us", "recompute_us")}), flush=True)
+    elif name == "sweep_scan":
+        # the same sweep's tail at L = 512 and recomputation at L = 4608 through the
+        # segment-parallel prefill only (3 calls each: both tensor-core passes and the scan)
+        r = sweep_run(dev, reps=1, seq=False, lengths=[512, 4608])
+        for row in r["rows"]:
+            print(json.dumps({k: row[k] for k in ("L", "tail_scan_us", "recompute_scan_us")}),
+                  flush=True)
     else:
         raise SystemExit(f"unknown case {name}")
     return 0
@@ -1586,7 +1595,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-extras", action="store_true",
                     help="skip TTFT arms, KV stress, e2e and CPU baseline")
-    ap.add_argument("--case", choices=["decode", "prefill", "kv", "ckpt", "long", "sweep"],
+    ap.add_argument("--case", choices=["decode", "prefill", "kv", "ckpt", "long", "sweep",
+                                       "sweep_scan"],
                     help="run one small standalone case for a profiler capture")
     ap.add_argument("--source-hashes", action="store_true",
                     help="print each profiled kernel's source hash (the key of profiles/*.txt rows)")
