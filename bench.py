@@ -89,7 +89,7 @@ KERNEL_SRC = {"gla_decode_kernel": "gla_decode.cu", "gla_chunked_tc_kernel": "gl
               "gla_recurrent_kernel": "gla_recurrent.cu", "restore_request_kernel": "restore_request.cu",
               "kv_scatter_kernel": "kv_scatter.cu", "kv_gather_kernel": "kv_scatter.cu",
               "kv_slices_kernel": "kv_scatter.cu", "slot_copy_kernel": "slot_copy.cu",
-              "gla_scan_kernel": "gla_scan.cu"}
+              "gla_scan_kernel": "gla_scan.cu", "gla_dstate_kernel": "gla_dstate.cu"}
 DTYPE = "bf16 q/k/v, fp32 log-gates; fp16 (fast) or tf32 (exact) MMA operands, fp32 accumulate, state and outputs"
 
 
@@ -114,14 +114,21 @@ def source_files(kernel: str) -> list:
     return files
 
 
+def _strip_comments(src: str) -> str:
+    """C/C++ source without its comments (string literals in these files hold no comment
+    markers), so that a documentation edit does not count as a kernel change."""
+    import re
+    return re.sub(r"/\*.*?\*/|//[^\n]*", "", src, flags=re.S)
+
+
 def source_hash(kernel: str) -> str:
     """First 12 hex digits of the SHA-256 of the kernel's source files (`source_files`: what
-    its machine code depends on): a profile row captured under another hash describes
-    another kernel."""
+    its machine code depends on), comments left out: a profile row captured under another
+    hash describes another kernel."""
     import hashlib
     h = hashlib.sha256()
     for f in source_files(kernel):
-        h.update(open(f, "rb").read())
+        h.update(_strip_comments(open(f).read()).encode())
     return h.hexdigest()[:12]
 
 

@@ -378,12 +378,12 @@ hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t 
  * Paper: as hs_linattn_prefill_from_state (Section 2.2, Section 4.1 and Table 2).
  * The recurrence is linear in the state, so over a segment [s,e) of the absolute
  * 64-token grid S_e = diag(G) S_s + dS with G = exp(sum of the segment's log-gates)
- * and dS the segment's state from the zero state.  Three launches: the tensor-core
- * kernel runs every segment as a problem of its own from the zero state (dS), an
- * elementwise scan chains S_{n+1} = G_n S_n + dS_n per (problem, head) and writes
- * the checkpoints and the final state, and the tensor-core kernel runs every
- * segment again from its start state S_n for the outputs.  A call with one problem
- * of 16 heads then occupies (segments x 16) CTAs instead of 16.
+ * and dS the segment's state from the zero state.  Three launches: a segment-state
+ * kernel computes every (segment, head)'s dS and G at once (tf32 tensor-core
+ * products), an elementwise scan chains S_{n+1} = G_n S_n + dS_n per (problem, head)
+ * and writes the checkpoints and the final state, and the tensor-core prefill kernel
+ * runs every segment again from its start state S_n for the outputs.  A call with
+ * one problem of 16 heads then occupies (segments x 16) CTAs instead of 16.
  *
  * Results: the outputs, final states and checkpoints of the same recurrence, within
  * the same accuracy as hs_linattn_prefill_from_state (the two are not bit-identical:

@@ -3,21 +3,24 @@
 // Over a problem's tail [pos0, pos0 + n), split into segments at the multiples of 64 of the
 // absolute position grid, the recurrence S_t = diag(g_t) S_{t-1} + k_t v_t^T is linear in
 // the state: for a segment of tokens [s, e),
-//     S_e = diag(G) S_s + dS,   G = prod_{s<=t<e} g_t = exp(sum_t a_t),
+//     S_e = diag(G) S_s + dS,   G = prod_{s<=t<e} g_t = 2^{sum_t a_t log2 e},
 // where dS is the segment's state when it starts from the zero state.  The first pass of the
-// prefill computes every segment's dS at once (each segment its own problem for the
-// tensor-core kernel); this kernel chains them: per (problem, head) and state element,
-// S_{n+1} = G_n S_n + dS_n over the segments in order, recording each segment's start state
-// S_n (the last pass computes the outputs from it), the checkpoint at every multiple of C
-// and the final state.  Every step is an elementwise fma, so a run resumed at a checkpoint
-// on the grid repeats the same operations from there: resumed and full computations agree
-// bit for bit.
+// prefill (gla_dstate.cu) computes every segment's dS and G at once; this kernel chains them:
+// per (problem, head) and state element, S_{n+1} = G_n S_n + dS_n over the segments in order,
+// recording each segment's start state S_n (the last pass computes the outputs from it), the
+// checkpoint at every multiple of C and the final state.  Every step is an elementwise fma,
+// so a run resumed at a checkpoint on the grid repeats the same operations from there:
+// resumed and full computations agree bit for bit.
 //
 // One CTA per (problem, head, block of 512 state elements); thread i owns four consecutive
-// elements of one key row d (a float4).  The D/4 lanes that share a row (a warp at D = 128,
-// a half-warp at D = 64) sum the row's log-gates over the segment (256/D tokens per lane, then
-// a butterfly, the same order in every lane).  The dS and log-gates of the next kPF segments
-// are loaded while the current one is applied.
+// elements (d, e..e+3) of one key row d (a float4), and the D/4 lanes of a row (a warp at
+// D = 128, a half-warp at D = 64) are consecutive.  The first pass leaves G_n of row d at
+// element (d, 0) of segment n's start-state block: the row's first lane, which owns that
+// element, reads it there, passes it to the row's other lanes with a shuffle and then
+// overwrites it with the start state.  The chain only streams: each thread copies its float4
+// of dS_n (the first lane also G_n) for the next kStages segments into its own slots of
+// shared-memory rings with cp.async (one commit group per segment, so that waiting for the
+// oldest group never waits for a newer copy), applies the oldest and refills its slots.
 #include "hs_internal.cuh"
 
 namespace hs {
@@ -25,16 +28,33 @@ namespace {
 
 constexpr int kThreads = 128;        // float4 per thread: 512 state elements per CTA
 constexpr int kChunk = 64;           // segments on the 64-token absolute grid
-constexpr int kPF = 4;               // segments loaded ahead
+constexpr int kStages = 16;          // segments whose dS and G are in flight
 
-// sum over the W lanes of an aligned group (a butterfly: the same order in every lane)
-template <int W>
-__device__ __forceinline__ float group_sum(float v)
+__device__ __forceinline__ void cp_async16(void *smem_dst, const void *gmem_src)
 {
-#pragma unroll
-    for (int o = W / 2; o > 0; o >>= 1)
-        v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                     (uint32_t)__cvta_generic_to_shared(smem_dst)),
+                 "l"(gmem_src)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cp_async4(void *smem_dst, const void *gmem_src)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                     (uint32_t)__cvta_generic_to_shared(smem_dst)),
+                 "l"(gmem_src)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit()
+{
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+// wait until at most kStages - 1 of this thread's commit groups are pending
+__device__ __forceinline__ void cp_async_wait_oldest()
+{
+    asm volatile("cp.async.wait_group %0;" ::"n"(kStages - 1) : "memory");
 }
 
 template <int D>
@@ -42,13 +62,16 @@ __global__ void __launch_bounds__(kThreads)
 gla_scan_kernel(const __grid_constant__ ScanParams p)
 {
     constexpr int BLOCKS = D * D / (4 * kThreads);   // CTAs per (problem, head)
+    __shared__ float4 sRing[kStages][kThreads];      // dS of the segments in flight
+    __shared__ float sGate[kStages][kThreads];       // their G (in a row's first lane)
+    constexpr int W = D / 4;                         // lanes per key row
+    const int lane = threadIdx.x & 31;
+    const bool row_lead = (lane & (W - 1)) == 0;
     const int bh = blockIdx.x / BLOCKS;
     const int blk = blockIdx.x - bh * BLOCKS;
     const int b = bh / p.n_heads;
     const int h = bh - b * p.n_heads;
-    const int lane = threadIdx.x & 31;
     const int f = (blk * kThreads + threadIdx.x) * 4;  // first of this thread's 4 elements
-    const int d = f / D;                               // its key row (one row per warp at D = 128)
     const int64_t pos0 = p.pos0[b];
     const int64_t end = pos0 + p.n_tokens[b];
     const int64_t hs_ = (int64_t)h * D * D + f;        // offset inside one [n_heads][D][D] state
@@ -58,75 +81,61 @@ gla_scan_kernel(const __grid_constant__ ScanParams p)
 
     float4 *st = reinterpret_cast<float4 *>(p.state + (int64_t)b * sstride + hs_);
     float4 S = *st;
-    // the sum of the log-gates of key row d over the tokens [s, e) of this problem
-    constexpr int W = D / 4;            // lanes per key row
-    constexpr int TPL = kChunk / W;     // tokens per lane
-    const int r = lane % W;
-    auto gate_sum = [&](int64_t s, int64_t e) -> float {
-        float v = 0.f;
-#pragma unroll
-        for (int j = 0; j < TPL; ++j) {
-            const int64_t t = s + r + W * j;
-            if (t < e) {
-                const int64_t row = (int64_t)p.row0[b] + (t - pos0);
-                v += p.log_g[(row * p.n_heads + h) * D + d];
-            }
-        }
-        return group_sum<W>(v);
-    };
-    // a ring of the next kPF segments' dS and log-gate sums, refilled as each is applied, so
-    // that the loads of later segments overlap the chain of fmas
     auto seg_end_of = [&](int64_t at) -> int64_t { return min(end, (at / kChunk + 1) * kChunk); };
-    float4 dq[kPF];
-    float aq[kPF];
-    int64_t ld_at = pos0;             // start of the next segment to load
+    // the rings: one commit group per segment (empty past the last), kStages in flight
+    int64_t ld_at = pos0;             // start of the next segment to copy
     int32_t ld_seg = p.seg_base[b];
-#pragma unroll
-    for (int j = 0; j < kPF; ++j) {
-        dq[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-        aq[j] = 0.f;
+    auto refill = [&](int slot) {
         if (ld_at < end) {
-            const int64_t e = seg_end_of(ld_at);
-            dq[j] = *reinterpret_cast<const float4 *>(p.dS + (int64_t)ld_seg * sstride + hs_);
-            aq[j] = gate_sum(ld_at, e);
-            ld_at = e;
+            const int64_t o = (int64_t)ld_seg * sstride + hs_;
+            cp_async16(&sRing[slot][threadIdx.x], p.dS + o);
+            if (row_lead)
+                cp_async4(&sGate[slot][threadIdx.x], p.Sn + o);
+            ld_at = seg_end_of(ld_at);
             ++ld_seg;
         }
-    }
+        cp_async_commit();
+    };
+    for (int j = 0; j < kStages; ++j)
+        refill(j);
     int64_t at = pos0;
     int32_t seg = p.seg_base[b];
+    // the next checkpoint position on the grid and its slot pointer, read one checkpoint
+    // ahead (only for positions within the call: the pointer array ends there)
+    int64_t next_ck = (C > 0 && p.ckpt_slots != nullptr) ? (pos0 / C + 1) * C : INT64_MAX;
+    int32_t ck = p.ck_base[b];
+    float *cs_next = next_ck <= end ? p.ckpt_slots[ck] : nullptr;
+    int slot = 0;
     while (at < end) {
-#pragma unroll
-        for (int j = 0; j < kPF; ++j) {
-            if (at < end) {
-                const int64_t e = seg_end_of(at);
-                *reinterpret_cast<float4 *>(p.Sn + (int64_t)seg * sstride + hs_) = S;
-                const float G = expf(aq[j]);
-                S.x = fmaf(G, S.x, dq[j].x);
-                S.y = fmaf(G, S.y, dq[j].y);
-                S.z = fmaf(G, S.z, dq[j].z);
-                S.w = fmaf(G, S.w, dq[j].w);
-                if (C > 0 && p.ckpt_slots != nullptr && e % C == 0) {
-                    float *slot = p.ckpt_slots[p.ck_base[b] + (e / C - pos0 / C - 1)];
-                    if (slot == nullptr || (reinterpret_cast<uintptr_t>(slot) & 15u) != 0) {
-                        if (threadIdx.x == 0 && blk == 0 && h == 0)
-                            report(p.d_err, slot == nullptr ? HS_DEVERR_NULL : HS_DEVERR_MISALIGNED);
-                    } else {
-                        *reinterpret_cast<float4 *>(slot + hs_) = S;
-                    }
-                }
-                if (ld_at < end) {
-                    const int64_t e2 = seg_end_of(ld_at);
-                    dq[j] = *reinterpret_cast<const float4 *>(p.dS + (int64_t)ld_seg * sstride + hs_);
-                    aq[j] = gate_sum(ld_at, e2);
-                    ld_at = e2;
-                    ++ld_seg;
-                }
-                at = e;
-                ++seg;
+        const int64_t e = seg_end_of(at);
+        cp_async_wait_oldest();
+        const float4 dq = sRing[slot][threadIdx.x];
+        const float G = __shfl_sync(0xffffffffu, row_lead ? sGate[slot][threadIdx.x] : 0.f,
+                                    lane & ~(W - 1));
+        // the start state replaces the gate the first pass left in the row's first float4
+        *reinterpret_cast<float4 *>(p.Sn + (int64_t)seg * sstride + hs_) = S;
+        S.x = fmaf(G, S.x, dq.x);
+        S.y = fmaf(G, S.y, dq.y);
+        S.z = fmaf(G, S.z, dq.z);
+        S.w = fmaf(G, S.w, dq.w);
+        if (e == next_ck) {
+            float *cs = cs_next;
+            next_ck += C;
+            if (next_ck <= end)
+                cs_next = p.ckpt_slots[++ck];
+            if (cs == nullptr || (reinterpret_cast<uintptr_t>(cs) & 15u) != 0) {
+                if (threadIdx.x == 0 && blk == 0 && h == 0)
+                    report(p.d_err, cs == nullptr ? HS_DEVERR_NULL : HS_DEVERR_MISALIGNED);
+            } else {
+                *reinterpret_cast<float4 *>(cs + hs_) = S;
             }
         }
+        refill(slot);     // after the slot is consumed: its next copies cannot overtake the reads
+        slot = slot + 1 == kStages ? 0 : slot + 1;
+        at = e;
+        ++seg;
     }
+    asm volatile("cp.async.wait_all;" ::: "memory");
     *st = S;
 }
 

@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cstring>
 
+#include "gla_dstate.cuh"
 #include "hs_internal.cuh"
 #include "hs_test.h"
 
@@ -427,8 +428,8 @@ static hs_status scan_check(const hs_linattn_shape *shp, const int64_t *pos0,
             return HS_ERR_UNSUPPORTED;   // token rows are 32-bit
         total += n_segments(pos0[b], n_tokens[b]);
     }
-    if (total > INT32_MAX)
-        return HS_ERR_UNSUPPORTED;
+    if (total * s.n_heads > INT32_MAX)
+        return HS_ERR_UNSUPPORTED;   // (segment, head) units are 32-bit
     *n_seg = total;
     return HS_OK;
 }
@@ -503,59 +504,76 @@ hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q
     if (ck > INT32_MAX)
         return HS_ERR_INVALID_ARG;
 
-    // one tensor-core pass over every segment as a problem of its own, at most HS_MAX_BATCH
-    // segments per launch: from the zero state, writing each segment's state into dS and no
-    // outputs; or from the scanned start states Sn, writing the outputs and no states
-    auto pass = [&](bool from_zero) -> hs_status {
-        hs::GlaParams p;
-        int32_t j = 0;
-        int64_t first = 0;
-        auto flush = [&]() -> hs_status {
-            if (j == 0)
-                return HS_OK;
-            p.batch = j;
-            p.state = (from_zero ? ws_dS : ws_Sn) + first * per;
-            const hs_status r = cuda_status(hs::launch_gla_chunked_tc(p, (int)D, stream));
-            first += j;
-            j = 0;
-            return r;
-        };
-        auto reset = [&]() {
-            std::memset(&p, 0, sizeof p);
-            p.q = q;
-            p.k = k;
-            p.v = v;
-            p.log_g = log_g;
-            p.o = from_zero ? nullptr : o;
-            p.d_err = d_err;
-            p.n_heads = s.n_heads;
-            p.zero_state = from_zero ? 1 : 0;
-            p.no_state_out = from_zero ? 0 : 1;
-        };
-        reset();
-        for (int32_t b = 0; b < s.batch; ++b) {
-            const int64_t end = pos0[b] + n_tokens[b];
-            for (int64_t at = pos0[b]; at < end;) {
-                const int64_t e = std::min<int64_t>(end, (at / HS_CHUNK + 1) * HS_CHUNK);
-                p.pos0[j] = at;
-                p.n_tokens[j] = (int32_t)(e - at);
-                p.row0[j] = (int32_t)((int64_t)b * s.max_tokens + (at - pos0[b]));
-                at = e;
-                if (++j == HS_MAX_BATCH) {
-                    const hs_status r = flush();
-                    if (r != HS_OK)
-                        return r;
-                    reset();
-                }
-            }
-        }
-        return flush();
-    };
-    if ((st = pass(true)) != HS_OK)
+    // every segment's state from the zero state (dS)
+    hs::DStateParams dp;
+    std::memset(&dp, 0, sizeof dp);
+    dp.k = k;
+    dp.v = v;
+    dp.log_g = log_g;
+    dp.dS = ws_dS;
+    dp.Sn = ws_Sn;
+    dp.d_err = d_err;
+    dp.batch = s.batch;
+    dp.n_heads = s.n_heads;
+    dp.n_units = (int32_t)(n_seg * s.n_heads);
+    for (int32_t b = 0; b < s.batch; ++b) {
+        dp.pos0[b] = sp.pos0[b];
+        dp.n_tokens[b] = sp.n_tokens[b];
+        dp.row0[b] = sp.row0[b];
+        dp.seg_base[b] = sp.seg_base[b];
+    }
+    int sms = 0;
+    if ((st = sm_count(&sms)) != HS_OK)
         return st;
+    const int grid = (int)std::min<int64_t>(dp.n_units, 2 * (int64_t)sms);
+    if ((st = cuda_status(hs::launch_gla_dstate(dp, (int)D, grid, stream))) != HS_OK)
+        return st;
+
+    // the scan: start states, checkpoints, final state
     if ((st = cuda_status(hs::launch_gla_scan(sp, (int)D, stream))) != HS_OK)
         return st;
-    return pass(false);
+
+    // the tensor-core kernel over every segment as a problem of its own from its start state
+    // Sn, at most HS_MAX_BATCH segments per launch, writing the outputs and no state
+    hs::GlaParams p;
+    int32_t j = 0;
+    int64_t first = 0;
+    auto reset = [&]() {
+        std::memset(&p, 0, sizeof p);
+        p.q = q;
+        p.k = k;
+        p.v = v;
+        p.log_g = log_g;
+        p.o = o;
+        p.d_err = d_err;
+        p.n_heads = s.n_heads;
+        p.no_state_out = 1;
+    };
+    auto flush = [&]() -> hs_status {
+        if (j == 0)
+            return HS_OK;
+        p.batch = j;
+        p.state = ws_Sn + first * per;
+        const hs_status r = cuda_status(hs::launch_gla_chunked_tc(p, (int)D, stream));
+        first += j;
+        j = 0;
+        reset();
+        return r;
+    };
+    reset();
+    for (int32_t b = 0; b < s.batch; ++b) {
+        const int64_t end = pos0[b] + n_tokens[b];
+        for (int64_t at = pos0[b]; at < end;) {
+            const int64_t e = std::min<int64_t>(end, (at / HS_CHUNK + 1) * HS_CHUNK);
+            p.pos0[j] = at;
+            p.n_tokens[j] = (int32_t)(e - at);
+            p.row0[j] = (int32_t)((int64_t)b * s.max_tokens + (at - pos0[b]));
+            at = e;
+            if (++j == HS_MAX_BATCH && (st = flush()) != HS_OK)
+                return st;
+        }
+    }
+    return flush();
 }
 
 hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t *q,

@@ -19,6 +19,10 @@ def test_kv_bytes_read_plus_write():
     assert bench.kv_bytes(48, 256, 65536) == 2 * 48 * 256 * 65536
 
 
+def test_source_hash_ignores_comments():
+    assert bench._strip_comments("a /* x\n y */ b // z\nc") == "a  b \nc"
+
+
 def test_source_hash_names_the_kernel_source():
     h = bench.source_hash("gla_decode_kernel<128>")
     assert len(h) == 12 and h == bench.source_hash("gla_decode_kernel@anything")
