@@ -583,12 +583,10 @@ cudaError_t launch_tc(const GlaParams &p, cudaStream_t s)
         !encode_rows<D>(&maps.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, p.v, inner, rows, 2) ||
         !encode_rows<D>(&maps.g, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, p.log_g, inner, rows, 4))
         return cudaErrorInvalidValue;
-    cudaError_t e = cudaFuncSetAttribute(gla_chunked_tc_kernel<D>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-    if (e != cudaSuccess)
-        return e;
+    static std::atomic<uint64_t> smem_set{0};
     const unsigned grid = (unsigned)p.batch * (unsigned)p.n_heads;
-    return launch_pdl(gla_chunked_tc_kernel<D>, dim3(grid), dim3(NT), SMEM_BYTES, s, p, maps);
+    return launch_pdl_big_smem(gla_chunked_tc_kernel<D>, dim3(grid), dim3(NT), SMEM_BYTES, s,
+                               smem_set, p, maps);
 }
 
 }  // namespace

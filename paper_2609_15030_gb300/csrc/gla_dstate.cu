@@ -6,8 +6,9 @@
 // tensor-core prefill applied to the zero state.
 //
 // One unit = one (segment, head).  All 256 threads stage the segment's k, v and log-gates
-// in shared memory with independent 16-byte loads (zeros past the segment's end, which leave
-// the results unchanged).  Then the 128 key-dim threads walk the 64 tokens backwards, keeping
+// in shared memory with cp.async (zeros past the segment's end, which leave the results
+// unchanged); a CTA stages its next unit as soon as the current one's operands are built, so
+// the copies overlap that unit's products and stores.  Then the 128 key-dim threads walk the 64 tokens backwards, keeping
 // Lam_last - Lam_j as a running sum of the later tokens' log2-gates, and write K^ rounded to
 // tf32 into a K-major operand (token = K), while the 128 value-dim threads put V^T into TMEM
 // (bf16 values, exact in tf32); one thread issues dS^T = V^T K^ as eight M = 128, N = d,
@@ -49,6 +50,15 @@ constexpr uint32_t kSmemBytes = 98304 + 1024;
 constexpr uint64_t kTimeoutNs = 1000000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
 
+// 16 bytes global -> shared, asynchronous; the first `n` bytes copied, the rest zero-filled
+__device__ __forceinline__ void cp_async16_zfill(void *smem_dst, const void *gmem_src, uint32_t n)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(
+                     (uint32_t)__cvta_generic_to_shared(smem_dst)),
+                 "l"(gmem_src), "r"(n)
+                 : "memory");
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 2)
 gla_dstate_kernel(const __grid_constant__ DStateParams p)
@@ -79,55 +89,59 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
     uint32_t ph = 0;
     bool aborted = false;
 
-    for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
-        const int g = u / p.n_heads;
-        const int h = u - g * p.n_heads;
+    // where unit u's segment lies: its (segment, head), token count and first element
+    struct Unit {
+        int g, h, L;
+        int64_t base;
+    };
+    auto unit = [&](int u) -> Unit {
+        Unit r;
+        r.g = u / p.n_heads;
+        r.h = u - r.g * p.n_heads;
         // the problem holding segment g: the last b with seg_base[b] <= g (problems without
         // tokens hold no segment and share the next one's seg_base)
         int lo = 0, hi = p.batch - 1;
         while (lo < hi) {
             const int mid = (lo + hi + 1) >> 1;
-            if (p.seg_base[mid] <= g)
+            if (p.seg_base[mid] <= r.g)
                 lo = mid;
             else
                 hi = mid - 1;
         }
-        const int b = lo;
-        const int64_t pos0 = p.pos0[b];
-        const int64_t chunk = pos0 / kChunk + (g - p.seg_base[b]);
+        const int64_t pos0 = p.pos0[lo];
+        const int64_t chunk = pos0 / kChunk + (r.g - p.seg_base[lo]);
         const int64_t s = max(pos0, chunk * kChunk);
-        const int L = (int)(min(pos0 + p.n_tokens[b], (chunk + 1) * kChunk) - s);
-        const int64_t base = ((int64_t)p.row0[b] + (s - pos0)) * tstride + (int64_t)h * D;
-
-        // stage the segment: token j < L of k, v (D/8 vectors each) and the log-gates (D/4
-        // vectors); tokens j >= L as zeros
-        {
-            constexpr int VK = D / 8, VA = D / 4;
-            const int4 zero = make_int4(0, 0, 0, 0);
-            int4 rk[64 * VK / kThreads], rv[64 * VK / kThreads], ra[64 * VA / kThreads];
+        r.L = (int)(min(pos0 + p.n_tokens[lo], (chunk + 1) * kChunk) - s);
+        r.base = ((int64_t)p.row0[lo] + (s - pos0)) * tstride + (int64_t)r.h * D;
+        return r;
+    };
+    // copy a unit's k, v (D/8 vectors per token) and log-gates (D/4) into the staging areas
+    // (tokens j >= L zero-filled: no bytes read), as one cp.async group of this thread
+    auto stage = [&](const Unit &w) {
+        constexpr int VK = D / 8, VA = D / 4;
 #pragma unroll
-            for (int x = 0; x < 64 * VK / kThreads; ++x) {
-                const int i = tid + x * kThreads, j = i / VK, c = i - j * VK;
-                const int64_t off = base + (int64_t)j * tstride + c * 8;
-                rk[x] = j < L ? __ldg(reinterpret_cast<const int4 *>(p.k + off)) : zero;
-                rv[x] = j < L ? __ldg(reinterpret_cast<const int4 *>(p.v + off)) : zero;
-            }
-#pragma unroll
-            for (int x = 0; x < 64 * VA / kThreads; ++x) {
-                const int i = tid + x * kThreads, j = i / VA, c = i - j * VA;
-                const int64_t off = base + (int64_t)j * tstride + c * 4;
-                ra[x] = j < L ? __ldg(reinterpret_cast<const int4 *>(p.log_g + off)) : zero;
-            }
-#pragma unroll
-            for (int x = 0; x < 64 * VK / kThreads; ++x) {
-                const int i = tid + x * kThreads;
-                reinterpret_cast<int4 *>(smem + OFF_K)[i] = rk[x];
-                reinterpret_cast<int4 *>(smem + OFF_V)[i] = rv[x];
-            }
-#pragma unroll
-            for (int x = 0; x < 64 * VA / kThreads; ++x)
-                reinterpret_cast<int4 *>(smem + OFF_A)[tid + x * kThreads] = ra[x];
+        for (int x = 0; x < 64 * VK / kThreads; ++x) {
+            const int i = tid + x * kThreads, j = i / VK, c = i - j * VK;
+            const int64_t off = w.base + (int64_t)min(j, w.L - 1) * tstride + c * 8;
+            const uint32_t n = j < w.L ? 16u : 0u;
+            cp_async16_zfill(smem + OFF_K + i * 16, p.k + off, n);
+            cp_async16_zfill(smem + OFF_V + i * 16, p.v + off, n);
         }
+#pragma unroll
+        for (int x = 0; x < 64 * VA / kThreads; ++x) {
+            const int i = tid + x * kThreads, j = i / VA, c = i - j * VA;
+            const int64_t off = w.base + (int64_t)min(j, w.L - 1) * tstride + c * 4;
+            cp_async16_zfill(smem + OFF_A + i * 16, p.log_g + off, j < w.L ? 16u : 0u);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+
+    Unit w = unit(blockIdx.x);
+    if ((int)blockIdx.x < p.n_units)
+        stage(w);
+    for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
+        const int g = w.g, h = w.h;
+        asm volatile("cp.async.wait_all;" ::: "memory");
         __syncthreads();
         if (warp < 4) {
             const int d = tid;
@@ -158,7 +172,7 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
             tmem_wait_st();
         }
         tc_fence_before();
-        __syncthreads();
+        __syncthreads();   // the operands are built: the staging areas are free
         if (tid == 0) {
             tc_fence_after();
 #pragma unroll
@@ -168,6 +182,11 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
                             idesc,
                             kk > 0);
             tc_commit(bar);
+        }
+        // the next unit's inputs arrive while this one's products and stores run
+        if (u + (int)gridDim.x < p.n_units) {
+            w = unit(u + gridDim.x);
+            stage(w);
         }
         aborted = __syncthreads_or(!mbar_wait_bounded(bar, ph, kTimeoutNs));
         if (aborted)
@@ -195,6 +214,7 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
         report(p.d_err, HS_DEVERR_TIMEOUT);
         mbar_wait_bounded(bar, ph, kTimeoutNs);   // the products in flight, before TMEM goes
     }
+    asm volatile("cp.async.wait_all;" ::: "memory");   // a staged next unit, after an abort
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
@@ -206,11 +226,9 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
 template <int D>
 cudaError_t launch_d(const DStateParams &p, int grid, cudaStream_t s)
 {
-    cudaError_t e = cudaFuncSetAttribute(gla_dstate_kernel<D>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-    if (e != cudaSuccess)
-        return e;
-    return launch_pdl(gla_dstate_kernel<D>, dim3(grid), dim3(kThreads), kSmemBytes, s, p);
+    static std::atomic<uint64_t> smem_set{0};
+    return launch_pdl_big_smem(gla_dstate_kernel<D>, dim3(grid), dim3(kThreads), kSmemBytes, s,
+                               smem_set, p);
 }
 
 }  // namespace

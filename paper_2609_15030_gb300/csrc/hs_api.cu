@@ -20,13 +20,20 @@ inline hs_status cuda_status(cudaError_t e)
     return e == cudaSuccess ? HS_OK : HS_ERR_CUDA;
 }
 
+// the current device's SM count, queried once per device
+std::atomic<int> g_sm_count[64];
+
 hs_status sm_count(int *out)
 {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess)
         return HS_ERR_CUDA;
+    if (dev >= 0 && dev < 64 && (*out = g_sm_count[dev].load(std::memory_order_relaxed)) > 0)
+        return HS_OK;
     if (cudaDeviceGetAttribute(out, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return HS_ERR_CUDA;
+    if (dev >= 0 && dev < 64)
+        g_sm_count[dev].store(*out, std::memory_order_relaxed);
     return HS_OK;
 }
 

@@ -1,6 +1,7 @@
 // Internal declarations shared by the library's translation units.
 #pragma once
 
+#include <atomic>
 #include <cstdint>
 #include <utility>
 #include <cuda_runtime.h>
@@ -50,6 +51,39 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
 }
 
 // First detected device-side problem wins; kernels never clear the word.
+// Launch a kernel that needs more than 48 KiB of dynamic shared memory.  Its limit is set
+// with cudaFuncSetAttribute on the first launch on each device (bit `dev` of `done`) instead
+// of on every call; if a launch still fails (the device's context was reset since), the
+// error is cleared, the limit set again and the launch retried once.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl_big_smem(void (*kernel)(KArgs...), dim3 grid, dim3 block,
+                                       size_t smem, cudaStream_t stream,
+                                       std::atomic<uint64_t> &done, Args &&...args)
+{
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return e;
+    const uint64_t bit = dev >= 0 && dev < 64 ? 1ull << dev : 0;
+    if (bit == 0 || (done.load(std::memory_order_acquire) & bit) == 0) {
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess)
+            return e;
+        done.fetch_or(bit, std::memory_order_acq_rel);
+        return launch_pdl(kernel, grid, block, smem, stream, std::forward<Args>(args)...);
+    }
+    e = launch_pdl(kernel, grid, block, smem, stream, args...);
+    if (e == cudaSuccess)
+        return e;
+    (void)cudaGetLastError();
+    done.fetch_and(~bit, std::memory_order_acq_rel);
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess)
+        return e;
+    done.fetch_or(bit, std::memory_order_acq_rel);
+    return launch_pdl(kernel, grid, block, smem, stream, std::forward<Args>(args)...);
+}
+
 __device__ __forceinline__ void report(int32_t *d_err, int32_t code)
 {
     if (d_err != nullptr)
