@@ -521,7 +521,7 @@ __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t t
     const int colhalf = (warp >> 2) & 1;
     const int e_own = (warp & 3) * 32 + lane;                  // TMEM lane = value dim e
 
-    if (ob == nullptr || !worker || (spare_issuer && warp == 8) || e_own >= D)
+    if (!worker || (spare_issuer && warp == 8) || e_own >= D)
         return;
     const int h0 = (spare_issuer && warp == 12) ? 0 : colhalf;
     const int h1 = (spare_issuer && warp == 12) ? 2 : colhalf + 1;
@@ -548,8 +548,7 @@ __device__ __forceinline__ void out_epilogue(uint32_t tmem, float *ob, int64_t t
 
 // ---- the state between global memory ([d][e], row = key dim) and TMEM (S^T, lane e) ----
 
-// (state warps) load a state into TMEM and record its largest |S| (float32) for the guard;
-// src == nullptr loads the zero state
+// (state warps) load a state into TMEM and record its largest |S| (float32) for the guard
 template <int D>
 __device__ __forceinline__ void state_load(uint8_t *smem, uint32_t tmem, const float *src)
 {
@@ -569,7 +568,7 @@ __device__ __forceinline__ void state_load(uint8_t *smem, uint32_t tmem, const f
             const int d0 = colhalf * CW + c0;
 #pragma unroll
             for (int x = 0; x < 32; ++x) {
-                r[x] = src != nullptr ? src[(int64_t)(d0 + x) * D + e_own] : 0.f;
+                r[x] = src[(int64_t)(d0 + x) * D + e_own];
                 m = fmaxf(m, fabsf(r[x]));
             }
             tmem_st32(tmem + lrow + TM_S + d0, r);
@@ -887,8 +886,6 @@ __device__ __forceinline__ void short_outputs(const uint8_t *smem, int L, float 
 {
     constexpr int NG = Geo<D>::NG;
     const float *part = reinterpret_cast<const float *>(smem);
-    if (ob == nullptr)
-        return;
     for (int idx = threadIdx.x; idx < L * D; idx += NT) {
         const int i = idx / D, e = idx % D;
         float sum = part[(i * NG) * D + e];

@@ -228,16 +228,14 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // largest magnitude.  The builders meanwhile stage and build the first segment.
     float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
     if (worker) {
-        state_load<D>(smem, tmem, p.zero_state ? nullptr : st_g);
+        state_load<D>(smem, tmem, st_g);
         tc_fence_before();
         bar_staters();
         tc_fence_after();
     }
 
-    // the output rows from local token t (nullptr: this launch writes no outputs)
-    auto outp = [&](int64_t t) -> float * {
-        return p.o != nullptr ? p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D : nullptr;
-    };
+    // the output rows from local token t
+    auto outp = [&](int64_t t) { return p.o + (((int64_t)p.row0[b] + t) * p.n_heads + h) * D; };
 
     // ---- a short segment (<= kShort tokens, staged inputs already waited for, no decay
     // pending): the per-token recurrence with the recurrent kernel's exact operation order

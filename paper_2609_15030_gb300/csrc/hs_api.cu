@@ -488,7 +488,6 @@ hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q
     // the scan's parameters (the original problems) and the segments' first rows
     hs::ScanParams sp;
     std::memset(&sp, 0, sizeof sp);
-    sp.log_g = log_g;
     sp.state = state;
     sp.dS = ws_dS;
     sp.Sn = ws_Sn;

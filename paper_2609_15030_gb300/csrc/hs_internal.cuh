@@ -104,10 +104,7 @@ struct GlaParams {
     int32_t n_heads;
     int32_t ckpt_interval;     // 0: none
     int32_t stall_for_test;    // tensor-core kernel only: one wait that nothing completes (failure-detection tests)
-    int32_t zero_state;        // tensor-core kernel only: start every problem from the zero state
-                               // (state is then only written)
     int32_t no_state_out;      // tensor-core kernel only: the final state is not written
-                               // (o == nullptr: no outputs are written either)
     int64_t pos0[HS_MAX_BATCH];
     int32_t n_tokens[HS_MAX_BATCH];
     int32_t ck_base[HS_MAX_BATCH];  // index of the problem's first slot in ckpt_slots
@@ -137,10 +134,10 @@ cudaError_t launch_slot_copy(const float *const *src, float *const *dst, int32_t
 // segment's decay factor per key dim, dS_n the segment's state from the zero state), recording
 // each segment's start state, the checkpoints and the final state.
 struct ScanParams {
-    const float *log_g;       // [rows][n_heads][d]
     float *state;             // [batch][n_heads][d][d]: in the state at pos0, out at pos0 + n
     const float *dS;          // [segments][n_heads][d][d]: each segment from the zero state
-    float *Sn;                // [segments][n_heads][d][d]: each segment's start state (written)
+    float *Sn;                // [segments][n_heads][d][d]: on entry each segment's decay G of
+                              // key row d at element (d, 0); on return its start state
     float *const *ckpt_slots; // as GlaParams
     int32_t *d_err;
     int32_t batch;
