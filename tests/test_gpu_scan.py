@@ -132,3 +132,72 @@ def test_scan_and_sequential_prefill_agree():
     o2, S2, _ = run_scan(inp, [1024], [512], S0, 512, dev)
     assert maxnorm_err(o2[0], o1[0], axes=(0, 2)) <= TOL
     assert maxnorm_err(S2, S1, axes=(2, 3)) <= TOL
+
+
+def test_scan_checkpoint_slot_errors_are_reported():
+    """A NULL or misaligned checkpoint slot read from the device pointer array: the scan
+    reports it in d_err (first error wins) and skips that slot's write."""
+    dev = device()
+    N, nH, d = 128, 2, 128
+    inp = gen_linear(8, 0, 1, N, nH, d, d)
+    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    state = torch.zeros((1, nH, d, d), device=dev)
+    o = torch.zeros((1, N, nH, d), device=dev)
+    slot = torch.zeros(nH * d * d + 4, device=dev)
+    shape = hs.make_shape(1, nH, d, d, N)
+    nb = hs.hs_linattn_scan_workspace_bytes(shape, [0], [N])
+    ws = torch.empty(nb // 4, device=dev)
+    for ptrs, code in (([slot.data_ptr() + 4, slot.data_ptr()], hs.HS_DEVERR_MISALIGNED),
+                       ([0, slot.data_ptr()], hs.HS_DEVERR_NULL)):
+        err = torch.zeros(1, dtype=torch.int32, device=dev)
+        state.zero_()
+        hs.hs_linattn_prefill_scan(shape, q, k, v, a, o, state, [0], [N], 64,
+                                   hs.ptr_array(ptrs, dev), ws, nb, err)
+        torch.cuda.synchronize()
+        assert err.item() == code
+
+
+def test_scan_graph_replay_equals_eager_call():
+    """The three launches of one call captured in a CUDA graph and replayed twice give the
+    bytes of the eager call (the workspace's stale contents do not matter either)."""
+    dev = device()
+    B, nH, d, T, C = 2, 8, 128, 448, 128
+    inp = gen_linear(12, 0, B, T, nH, d, d, "uniform")
+    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
+    S0 = torch.from_numpy(gen_state(12, 1, B, nH, d, d)).to(dev)
+    pos0, n = [256, 37], [448, 300]
+    shape = hs.make_shape(B, nH, d, d, T)
+    nck = hs.hs_linattn_num_checkpoints(pos0, n, C)
+    state = torch.empty_like(S0)
+    o = torch.empty((B, T, nH, d), device=dev)
+    slots = torch.empty((nck, nH, d, d), device=dev)
+    ptrs = hs.ptr_array([slots[i] for i in range(nck)], dev)
+    nb = hs.hs_linattn_scan_workspace_bytes(shape, pos0, n)
+    ws = torch.empty(nb // 4, device=dev)
+    s = torch.cuda.Stream(dev)
+
+    def reset():
+        state.copy_(S0)
+        o.fill_(float("nan"))
+        slots.fill_(float("nan"))
+        ws.fill_(float("nan"))
+        torch.cuda.synchronize()
+
+    def bits():
+        return [t.view(torch.int32).cpu().numpy() for t in (o, state, slots)]
+
+    reset()
+    hs.hs_linattn_prefill_scan(shape, q, k, v, a, o, state, pos0, n, C, ptrs, ws, nb, None,
+                               s.cuda_stream)
+    torch.cuda.synchronize()
+    ref = bits()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s, capture_error_mode="relaxed"):
+        hs.hs_linattn_prefill_scan(shape, q, k, v, a, o, state, pos0, n, C, ptrs, ws, nb, None,
+                                   torch.cuda.current_stream(dev).cuda_stream)
+    for _ in range(2):
+        reset()
+        g.replay()
+        torch.cuda.synchronize()
+        for x, y in zip(bits(), ref):
+            assert np.array_equal(x, y)
