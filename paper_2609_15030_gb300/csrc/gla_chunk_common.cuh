@@ -801,7 +801,8 @@ __device__ __forceinline__ void fast_issue_sq(uint32_t tmem, uint32_t sb, int pa
 // (K-major there, K = key dim); read with N = key dim contiguous it is the MN-major B operand
 // of the state update: 64-dim blocks 8 KiB apart (leading byte offset), 8-token row groups
 // 1 KiB apart (stride byte offset), 16 tokens = 2 KiB per step.
-template <int D>
+// (WITH_STATE false: D_O only, for launches that discard the state)
+template <int D, bool WITH_STATE = true>
 __device__ __forceinline__ void fast_issue_update(uint32_t tmem, uint32_t sb, int par)
 {
     const uint32_t setb = sb + (uint32_t)par * SET_BYTES;
@@ -810,8 +811,9 @@ __device__ __forceinline__ void fast_issue_update(uint32_t tmem, uint32_t sb, in
     for (int kk = 0; kk < CH / 16; ++kk) {
         mma_f16_ts(tmem + (par ? Geo<D>::O1 : TM_O0), vt + kk * 8,
                    sdesc_sw128(setb + S_AH + kk * 32, 16, 1024), IDF_N64, 1);
-        mma_f16_ts(tmem + TM_S, vt + kk * 8, sdesc_sw128(setb + S_KH + kk * 2048, 8192, 1024),
-                   Geo<D>::IDF_ST, 1);
+        if (WITH_STATE)
+            mma_f16_ts(tmem + TM_S, vt + kk * 8, sdesc_sw128(setb + S_KH + kk * 2048, 8192, 1024),
+                       Geo<D>::IDF_ST, 1);
     }
 }
 

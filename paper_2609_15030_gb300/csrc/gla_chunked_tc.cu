@@ -55,7 +55,12 @@ namespace {
 using namespace ptx;
 using namespace gck;
 
-template <int D>
+// RESTART: the output pass of the segment-parallel prefill.  Every segment of a problem
+// starts from its own start state (segment k of problem b from state slot ck_base[b] + k of
+// p.state) instead of the state the previous segment leaves, and the run of fast segments
+// ends after one segment, so that a segment's outputs do not depend on which other segments
+// share its CTA.
+template <int D, bool RESTART>
 __global__ void __launch_bounds__(NT, 1)
 gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant__ TmaMaps maps)
 {
@@ -226,7 +231,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
 
     // incoming state -> TMEM (state warps), transposed: S^T[e][d] = state[d][e]; its
     // largest magnitude.  The builders meanwhile stage and build the first segment.
-    float *st_g = p.state + ((int64_t)b * p.n_heads + h) * D * D;
+    float *st_g = p.state + ((int64_t)(RESTART ? p.ck_base[b] : b) * p.n_heads + h) * D * D;
     if (worker) {
         state_load<D>(smem, tmem, st_g);
         tc_fence_before();
@@ -360,7 +365,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             if (!wait_group(1, kLoader, bar_go, ph_go))
                 return;
-            if (sMisc[2] == 0 || !next_long)
+            if (RESTART || sMisc[2] == 0 || !next_long)
                 return;
             rpos += L;
             rtok += L;
@@ -421,7 +426,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 return;
             if (tid == kIssuer) {
                 tc_fence_after();
-                fast_issue_update<D>(tmem, sb, par);
+                fast_issue_update<D, !RESTART>(tmem, sb, par);   // RESTART: S is discarded
                 tc_commit(bar_o);
             }
             pend = true;
@@ -434,7 +439,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             rtok += L;
             par ^= 1;
             ++kseq;
-            if (!is_long(rpos))
+            if (RESTART || !is_long(rpos))
                 break;
             // the builders' next segment, and the decision on it: the state it starts from is
             // bounded by the fp16 copy's largest |S| at this segment's start plus this segment's
@@ -456,7 +461,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (pend) {
             if (!wait_group(2, kIssuer, bar_o, ph_o))
                 return;
-            state_pass<D>(smem, tmem, pend_g, ckpt_slot(pend_end), false);
+            if (!RESTART)   // RESTART: no checkpoint, and the next segment loads its own state
+                state_pass<D>(smem, tmem, pend_g, ckpt_slot(pend_end), false);
             out_epilogue<D>(tmem, outp(pend_tok), tstride, pend_L, pend_par, false);
             tc_fence_before();
             if (!sync_group(2))
@@ -479,7 +485,16 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     }
 
     int64_t pos = pos0, tok = 0;
+    int seg_k = 0;   // RESTART: segments of this problem done
     while (!aborted && pos < end) {
+        if (RESTART && seg_k > 0 && worker) {
+            // this segment's own start state (the previous segment's state is not used)
+            state_load<D>(smem, tmem, st_g + (int64_t)seg_k * p.n_heads * D * D);
+            tc_fence_before();
+            bar_staters();
+            tc_fence_after();
+        }
+        ++seg_k;
         const int L = seg_len(pos);
         if (L <= kShort) {
             // a leading or trailing short segment (its inputs are staged or in flight)
@@ -561,7 +576,7 @@ bool gla_chunked_tc_supported(int d)
 
 namespace {
 
-template <int D>
+template <int D, bool RESTART>
 cudaError_t launch_tc(const GlaParams &p, cudaStream_t s)
 {
     TmaMaps maps;
@@ -583,7 +598,7 @@ cudaError_t launch_tc(const GlaParams &p, cudaStream_t s)
         return cudaErrorInvalidValue;
     static std::atomic<uint64_t> smem_set{0};
     const unsigned grid = (unsigned)p.batch * (unsigned)p.n_heads;
-    return launch_pdl_big_smem(gla_chunked_tc_kernel<D>, dim3(grid), dim3(NT), SMEM_BYTES, s,
+    return launch_pdl_big_smem(gla_chunked_tc_kernel<D, RESTART>, dim3(grid), dim3(NT), SMEM_BYTES, s,
                                smem_set, p, maps);
 }
 
@@ -592,9 +607,18 @@ cudaError_t launch_tc(const GlaParams &p, cudaStream_t s)
 cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s)
 {
     if (d == 128)
-        return launch_tc<128>(p, s);
+        return launch_tc<128, false>(p, s);
     if (d == 64)
-        return launch_tc<64>(p, s);
+        return launch_tc<64, false>(p, s);
+    return cudaErrorNotSupported;
+}
+
+cudaError_t launch_gla_chunked_tc_restart(const GlaParams &p, int d, cudaStream_t s)
+{
+    if (d == 128)
+        return launch_tc<128, true>(p, s);
+    if (d == 64)
+        return launch_tc<64, true>(p, s);
     return cudaErrorNotSupported;
 }
 

@@ -539,11 +539,13 @@ hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q
     if ((st = cuda_status(hs::launch_gla_scan(sp, (int)D, stream))) != HS_OK)
         return st;
 
-    // the tensor-core kernel over every segment as a problem of its own from its start state
-    // Sn, at most HS_MAX_BATCH segments per launch, writing the outputs and no state
+    // the tensor-core kernel over every segment from its start state Sn, writing the outputs
+    // and no state.  Consecutive segments of a problem are grouped into spans, one CTA per
+    // (span, head), about one CTA per SM in all; each segment restarts from its own start
+    // state, so the grouping changes no result.  At most HS_MAX_BATCH spans per launch.
+    const int64_t per_span = std::max<int64_t>(1, (n_seg * s.n_heads + sms - 1) / sms);
     hs::GlaParams p;
     int32_t j = 0;
-    int64_t first = 0;
     auto reset = [&]() {
         std::memset(&p, 0, sizeof p);
         p.q = q;
@@ -551,6 +553,7 @@ hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q
         p.v = v;
         p.log_g = log_g;
         p.o = o;
+        p.state = ws_Sn;
         p.d_err = d_err;
         p.n_heads = s.n_heads;
         p.no_state_out = 1;
@@ -559,9 +562,7 @@ hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q
         if (j == 0)
             return HS_OK;
         p.batch = j;
-        p.state = ws_Sn + first * per;
-        const hs_status r = cuda_status(hs::launch_gla_chunked_tc(p, (int)D, stream));
-        first += j;
+        const hs_status r = cuda_status(hs::launch_gla_chunked_tc_restart(p, (int)D, stream));
         j = 0;
         reset();
         return r;
@@ -569,11 +570,19 @@ hs_status hs_linattn_prefill_scan(const hs_linattn_shape *shp, const uint16_t *q
     reset();
     for (int32_t b = 0; b < s.batch; ++b) {
         const int64_t end = pos0[b] + n_tokens[b];
+        int64_t seg_i = sp.seg_base[b];
         for (int64_t at = pos0[b]; at < end;) {
-            const int64_t e = std::min<int64_t>(end, (at / HS_CHUNK + 1) * HS_CHUNK);
+            // a span of up to per_span segments from `at`
+            int64_t e = at, n = 0;
+            while (e < end && n < per_span) {
+                e = std::min<int64_t>(end, (e / HS_CHUNK + 1) * HS_CHUNK);
+                ++n;
+            }
             p.pos0[j] = at;
             p.n_tokens[j] = (int32_t)(e - at);
             p.row0[j] = (int32_t)((int64_t)b * s.max_tokens + (at - pos0[b]));
+            p.ck_base[j] = (int32_t)seg_i;
+            seg_i += n;
             at = e;
             if (++j == HS_MAX_BATCH && (st = flush()) != HS_OK)
                 return st;

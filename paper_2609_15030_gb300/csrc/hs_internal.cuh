@@ -107,7 +107,9 @@ struct GlaParams {
     int32_t no_state_out;      // tensor-core kernel only: the final state is not written
     int64_t pos0[HS_MAX_BATCH];
     int32_t n_tokens[HS_MAX_BATCH];
-    int32_t ck_base[HS_MAX_BATCH];  // index of the problem's first slot in ckpt_slots
+    int32_t ck_base[HS_MAX_BATCH];  // index of the problem's first slot in ckpt_slots; in the
+                                    // restart launch (no checkpoints), of its first segment's
+                                    // start state in state
     int32_t row0[HS_MAX_BATCH];     // token row of the problem's first token in q/k/v/log_g/o
 };
 
@@ -153,6 +155,8 @@ cudaError_t launch_gla_scan(const ScanParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_recurrent(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_decode(const GlaParams &p, int d, cudaStream_t s);
 cudaError_t launch_gla_chunked_tc(const GlaParams &p, int d, cudaStream_t s);
+// every segment from its own start state (see the kernel); ckpt_slots must be nullptr
+cudaError_t launch_gla_chunked_tc_restart(const GlaParams &p, int d, cudaStream_t s);
 bool gla_chunked_tc_supported(int d);
 
 }  // namespace hs

@@ -82,10 +82,12 @@ def test_scan_matches_the_oracle(name):
 
 
 @pytest.mark.parametrize("d,N,c,C", [(128, 1024, 512, 512), (128, 700, 256, 128),
-                                     (64, 512, 192, 64)])
+                                     (64, 512, 192, 64), (128, 4608, 4096, 512)])
 def test_scan_resume_equals_its_recompute_bitwise(d, N, c, C):
     """The scan's full recomputation of [0,N) against its own resume from the checkpoint it
-    emitted at c: outputs of [c,N), the final state and the later checkpoints, bit for bit."""
+    emitted at c: outputs of [c,N), the final state and the later checkpoints, bit for bit.
+    At N = 4608 the recomputation's output pass gives each CTA two segments and the resume's
+    one, so this also checks that grouping segments changes no output."""
     dev = device()
     inp = gen_linear(N + d, 0, 1, N, 4, d, d, "uniform")
     o_f, S_f, ck_f = run_scan(inp, [0], [N], None, C, dev)
