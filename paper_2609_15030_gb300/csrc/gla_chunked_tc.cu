@@ -57,9 +57,9 @@ using namespace gck;
 
 // RESTART: the output pass of the segment-parallel prefill.  Every segment of a problem
 // starts from its own start state (segment k of problem b from state slot ck_base[b] + k of
-// p.state) instead of the state the previous segment leaves, and the run of fast segments
-// ends after one segment, so that a segment's outputs do not depend on which other segments
-// share its CTA.
+// p.state) instead of the state the previous segment leaves, and decides its path on that
+// state as the first segment of a run does, so that a segment's outputs do not depend on
+// which other segments share its CTA; no state or checkpoint is written.
 template <int D, bool RESTART>
 __global__ void __launch_bounds__(NT, 1)
 gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant__ TmaMaps maps)
@@ -365,7 +365,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             }
             if (!wait_group(1, kLoader, bar_go, ph_go))
                 return;
-            if (RESTART || sMisc[2] == 0 || !next_long)
+            if (sMisc[2] == 0 || !next_long)
                 return;
             rpos += L;
             rtok += L;
@@ -426,7 +426,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                 return;
             if (tid == kIssuer) {
                 tc_fence_after();
-                fast_issue_update<D, !RESTART>(tmem, sb, par);   // RESTART: S is discarded
+                fast_issue_update<D>(tmem, sb, par);
                 tc_commit(bar_o);
             }
             pend = true;
@@ -439,7 +439,7 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
             rtok += L;
             par ^= 1;
             ++kseq;
-            if (RESTART || !is_long(rpos))
+            if (!is_long(rpos))
                 break;
             // the builders' next segment, and the decision on it: the state it starts from is
             // bounded by the fp16 copy's largest |S| at this segment's start plus this segment's
@@ -461,8 +461,104 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         if (pend) {
             if (!wait_group(2, kIssuer, bar_o, ph_o))
                 return;
-            if (!RESTART)   // RESTART: no checkpoint, and the next segment loads its own state
-                state_pass<D>(smem, tmem, pend_g, ckpt_slot(pend_end), false);
+            state_pass<D>(smem, tmem, pend_g, ckpt_slot(pend_end), false);
+            out_epilogue<D>(tmem, outp(pend_tok), tstride, pend_L, pend_par, false);
+            tc_fence_before();
+            if (!sync_group(2))
+                return;
+        }
+        if (tid == kIssuer) {
+            sMisc[3] = stop;
+            sRun[0] = rpos;
+            sRun[1] = rtok;
+        }
+    };
+
+    // RESTART: the state warps' side of a run in which every segment decides on, and is
+    // computed from, its own start state, loaded before its decision (the first segment's is
+    // loaded before the run); the builders' side is builder_run, unchanged.  No product reads
+    // the float32 state in TMEM here (the state update is skipped and D_O reads the fp16 copy),
+    // so the next segment's state is loaded while the previous segment's products run.
+    int loaded = 0;   // index of the segment whose start state is in TMEM (state warps)
+    auto seg_idx = [&](int64_t at) -> int { return (int)(at / CH - pos0 / CH); };
+    auto state_run_restart = [&](int64_t rpos, int64_t rtok) {
+        int par = 0;
+        bool pend = false;
+        uint32_t stop = 0;   // 0 done or short segment, 1 exact
+        int pend_par = 0, pend_L = 0;
+        int64_t pend_tok = 0;
+        while (true) {
+            const int L = seg_len(rpos);
+            if (!wait_group(2, kIssuer, bar_built, ph_built))
+                return;
+            if (loaded != seg_idx(rpos)) {
+                state_load<D>(smem, tmem, st_g + (int64_t)seg_idx(rpos) * p.n_heads * D * D);
+                loaded = seg_idx(rpos);
+            }
+            // the loaded state (its TMEM columns and its largest |S|) visible to the group
+            tc_fence_before();
+            if (!sync_group(2))
+                return;
+            tc_fence_after();
+            bool state_ok;
+            const bool fast = guard(state_max(), state_ok) && state_ok;
+            if (tid == kIssuer) {
+                sMisc[2] = fast ? 1u : 0u;
+                if (!fast)
+                    mbar_arrive(bar_go);
+            }
+            if (!fast) {
+                // the exact path takes this segment: its (unused) D_A product drained first
+                stop = 1;
+                if (!(par ? wait_group(2, kIssuer, bar_a1, ph_a1) : wait_group(2, kIssuer, bar_a, ph_a0)))
+                    return;
+                break;
+            }
+            if (pend && !wait_group(2, kIssuer, bar_o, ph_o))
+                return;
+            // the products of the previous segment are complete: its operand set is free
+            if (tid == kIssuer)
+                mbar_arrive(bar_go);
+            state_pass<D>(smem, tmem, -1, nullptr, true);   // the fp16 copy of S for D_O
+            tc_fence_before();
+            if (!sync_group(2))
+                return;
+            if (tid == kIssuer) {
+                tc_fence_after();
+                fast_issue_sq<D>(tmem, sb, par);
+            }
+            if (pend)
+                out_epilogue<D>(tmem, outp(pend_tok), tstride, pend_L, pend_par, true);
+            if (!(par ? wait_group(2, kIssuer, bar_a1, ph_a1) : wait_group(2, kIssuer, bar_a, ph_a0)))
+                return;
+            a_build<D>(smem, tmem, par);
+            fence_proxy_async_smem();
+            tc_fence_before();
+            if (!sync_group(2))
+                return;
+            if (tid == kIssuer) {
+                tc_fence_after();
+                fast_issue_update<D, false>(tmem, sb, par);   // D_O only: the state is discarded
+                tc_commit(bar_o);
+            }
+            pend = true;
+            pend_par = par;
+            pend_tok = rtok;
+            pend_L = L;
+            rpos += L;
+            rtok += L;
+            par ^= 1;
+            ++kseq;
+            if (!is_long(rpos))
+                break;
+            // the next segment's start state, while this segment's products run and the
+            // builders build it (this segment's fp16 copy is made: TMEM S is free)
+            state_load<D>(smem, tmem, st_g + (int64_t)seg_idx(rpos) * p.n_heads * D * D);
+            loaded = seg_idx(rpos);
+        }
+        if (pend) {
+            if (!wait_group(2, kIssuer, bar_o, ph_o))
+                return;
             out_epilogue<D>(tmem, outp(pend_tok), tstride, pend_L, pend_par, false);
             tc_fence_before();
             if (!sync_group(2))
@@ -485,16 +581,15 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     }
 
     int64_t pos = pos0, tok = 0;
-    int seg_k = 0;   // RESTART: segments of this problem done
     while (!aborted && pos < end) {
-        if (RESTART && seg_k > 0 && worker) {
+        if (RESTART && worker && loaded != seg_idx(pos)) {
             // this segment's own start state (the previous segment's state is not used)
-            state_load<D>(smem, tmem, st_g + (int64_t)seg_k * p.n_heads * D * D);
+            state_load<D>(smem, tmem, st_g + (int64_t)seg_idx(pos) * p.n_heads * D * D);
             tc_fence_before();
             bar_staters();
             tc_fence_after();
+            loaded = seg_idx(pos);
         }
-        ++seg_k;
         const int L = seg_len(pos);
         if (L <= kShort) {
             // a leading or trailing short segment (its inputs are staged or in flight)
@@ -507,6 +602,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
         }
         if (builder)
             builder_run(pos, tok);
+        else if constexpr (RESTART)
+            state_run_restart(pos, tok);
         else
             state_run(pos, tok);
         if (!sync_all())
