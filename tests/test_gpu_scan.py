@@ -203,3 +203,27 @@ def test_scan_graph_replay_equals_eager_call():
         torch.cuda.synchronize()
         for x, y in zip(bits(), ref):
             assert np.array_equal(x, y)
+
+
+def test_scan_exact_segments_inside_spans():
+    """Segments that take the exact path (strong decay, a zero gate) in the middle of the
+    output pass's multi-segment spans: the oracle bar, and the resume from a checkpoint
+    (two segments per CTA) equal to the recomputation (three per CTA) bit for bit."""
+    dev = device()
+    B, nH, d, N, C, c = 2, 4, 128, 2560, 512, 1024
+    inp = gen_linear(41, 0, B, N, nH, d, d, "uniform")
+    a = inp.a.copy()
+    a[0, 600:700] = -1.2          # strong decay over two chunks (exact path)
+    a[0, 1500] = -1e4             # a zero gate after the resume point
+    a[1, 1100:1180] = -1.2
+    inp = type(inp)(inp.q, inp.k, inp.v, a)
+    o_f, S_f, ck_f = run_scan(inp, [0, 0], [N, N], None, C, dev)
+    _check_oracle(inp, [0, 0], [N, N], None, C, (o_f, S_f, ck_f))
+    m = c // C - 1
+    sub = type(inp)(*(x[:, c:N].copy() for x in (inp.q, inp.k, inp.v, inp.a)))
+    S_c = np.stack([ck_f[b][m] for b in range(B)])
+    o_r, S_r, ck_r = run_scan(sub, [c, c], [N - c, N - c], S_c, C, dev)
+    assert np.array_equal(o_r.view(np.uint32), o_f[:, c:N].view(np.uint32))
+    assert np.array_equal(S_r.view(np.uint32), S_f.view(np.uint32))
+    for b in range(B):
+        assert np.array_equal(ck_r[b].view(np.uint32), ck_f[b][m + 1:].view(np.uint32))
