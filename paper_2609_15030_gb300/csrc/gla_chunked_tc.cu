@@ -14,19 +14,23 @@
 //
 // One CTA owns one (problem, head) and walks its segments in order; the
 // float32 state lives in tensor memory (TMEM) for the whole call, stored
-// transposed (lane = value dim e, column = key dim d).
+// transposed (lane = value dim e, column = key dim d).  (The RESTART
+// instantiation, the output pass of the segment-parallel prefill, instead
+// starts every segment from its own start state; see the kernel.)
 //
-// Fast chunks run three kind::f16 MMA groups with fp16 operands and float32
+// Fast chunks run kind::f16 MMA groups with fp16 operands and float32
 // accumulators:  D_O = S^T Q~^T (A operand: an fp16 copy of S^T in TMEM),
-// D_A = Q~ K~^T, then [D_O | S^T] += V^T [A ; K~^T]^T as one N=192 product
-// (V^T in TMEM).  fp16 keeps the 10-bit mantissa of tf32 but halves the
-// instructions (K = 16 per MMA).  The CTA's 16 warps form two groups in a
-// pipeline over two alternating operand sets: while the eight state warps
-// finish chunk c (the state pass, which applies the pending decay 2^{Lam_last},
-// writes a due checkpoint and refreshes the fp16 copy of S^T; the causal mask;
-// the output epilogue) the eight builder warps stage chunk c+1 and build its
-// operands (cumulative decay scan, Q~, K~, K~^T, V^T).  The first builder thread
-// issues the TMA copies and D_A, the first state thread the other MMAs.
+// D_A = Q~ K~^T, then per 16 tokens D_O += V^T A^T (N = 64) and S^T += V^T K~
+// (N = D, the K~ tile read MN-major), V^T in TMEM.  fp16 keeps the 10-bit
+// mantissa of tf32 but halves the instructions (K = 16 per MMA).  The CTA's
+// 16 warps form two groups in a pipeline over two alternating operand sets:
+// while the eight state warps finish chunk c (the state pass, which applies
+// the pending decay 2^{Lam_last}, writes a due checkpoint and refreshes the
+// fp16 copy of S^T; the causal mask with each token's own score summed in
+// float32 on the diagonal; the output epilogue) the eight builder warps stage
+// chunk c+1 and build its operands (cumulative decay scan, Q~, K~, V^T).  The
+// first builder thread issues the TMA copies and D_A, the first state thread
+// the other MMAs.
 //
 // A chunk is fast only if every fp16 operand provably stays below 2^15 in
 // magnitude (|q|, |v|, |K~|, the bound 128 max|q| max|k| on |A|, and a bound
