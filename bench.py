@@ -116,9 +116,10 @@ def source_files(kernel: str) -> list:
 
 def _strip_comments(src: str) -> str:
     """C/C++ source without its comments (string literals in these files hold no comment
-    markers), so that a documentation edit does not count as a kernel change."""
+    markers) and with every run of whitespace made one space, so that a documentation or
+    layout edit does not count as a kernel change."""
     import re
-    return re.sub(r"/\*.*?\*/|//[^\n]*", "", src, flags=re.S)
+    return re.sub(r"\s+", " ", re.sub(r"/\*.*?\*/|//[^\n]*", "", src, flags=re.S)).strip()
 
 
 def source_hash(kernel: str) -> str:

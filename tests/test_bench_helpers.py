@@ -20,7 +20,8 @@ def test_kv_bytes_read_plus_write():
 
 
 def test_source_hash_ignores_comments():
-    assert bench._strip_comments("a /* x\n y */ b // z\nc") == "a  b \nc"
+    assert bench._strip_comments("a /* x\n y */ b // z\nc") == "a b c"
+    assert bench._strip_comments("a\n// one\n// two\nb") == bench._strip_comments("a // one\nb")
 
 
 def test_source_hash_names_the_kernel_source():
