@@ -94,10 +94,10 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
         int g, h, L;
         int64_t base;
     };
-    auto unit = [&](int u) -> Unit {
+    auto unit = [&](int64_t u) -> Unit {
         Unit r;
-        r.g = u / p.n_heads;
-        r.h = u - r.g * p.n_heads;
+        r.g = (int)(u / p.n_heads);
+        r.h = (int)(u - (int64_t)r.g * p.n_heads);
         // the problem holding segment g: the last b with seg_base[b] <= g (problems without
         // tokens hold no segment and share the next one's seg_base)
         int lo = 0, hi = p.batch - 1;
@@ -137,9 +137,9 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
     };
 
     Unit w = unit(blockIdx.x);
-    if ((int)blockIdx.x < p.n_units)
+    if ((int64_t)blockIdx.x < p.n_units)
         stage(w);
-    for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
+    for (int64_t u = blockIdx.x; u < p.n_units; u += gridDim.x) {
         const int g = w.g, h = w.h;
         asm volatile("cp.async.wait_all;" ::: "memory");
         __syncthreads();
@@ -184,7 +184,7 @@ gla_dstate_kernel(const __grid_constant__ DStateParams p)
             tc_commit(bar);
         }
         // the next unit's inputs arrive while this one's products and stores run
-        if (u + (int)gridDim.x < p.n_units) {
+        if (u + gridDim.x < p.n_units) {
             w = unit(u + gridDim.x);
             stage(w);
         }
