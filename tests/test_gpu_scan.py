@@ -12,34 +12,9 @@ import torch
 import oracle
 import paper_2609_15030_gb300 as hs
 from hs_inputs import gen_linear, gen_state
-from tests.gpu_helpers import TOL, device, maxnorm_err, to_dev
+from tests.gpu_helpers import TOL, device, maxnorm_err, run_scan_prefill as run_scan, to_dev
 
 pytestmark = pytest.mark.gpu
-
-
-def run_scan(inp, pos0, n_tokens, S0, C, dev, kernel=hs.HS_LINATTN_AUTO):
-    """hs_linattn_prefill_scan on numpy inputs; returns numpy (o, S, checkpoint list)."""
-    q, k, v, a = (to_dev(x, dev) for x in (inp.q, inp.k, inp.v, inp.a))
-    B, T, nH, d = inp.q.shape
-    state = to_dev(np.zeros((B, nH, d, d), np.float32) if S0 is None
-                   else np.asarray(S0, np.float32), dev)
-    o = torch.full((B, T, nH, d), float("nan"), device=dev)
-    nck = hs.hs_linattn_num_checkpoints(pos0, n_tokens, C)
-    slots = torch.full((max(nck, 1), nH, d, d), float("nan"), device=dev)
-    ptrs = hs.ptr_array([slots[i] for i in range(nck)], dev) if nck else None
-    err = torch.zeros(1, dtype=torch.int32, device=dev)
-    shape = hs.make_shape(B, nH, d, d, T, kernel)
-    nb = hs.hs_linattn_scan_workspace_bytes(shape, pos0, n_tokens)
-    ws = torch.full((max(nb // 4, 4),), float("nan"), device=dev)   # stale contents must not matter
-    hs.hs_linattn_prefill_scan(shape, q, k, v, a, o, state, pos0, n_tokens, C, ptrs, ws, nb, err)
-    torch.cuda.synchronize()
-    assert int(err.item()) == 0
-    cks, i = [], 0
-    for b in range(B):
-        m = 0 if C == 0 or n_tokens[b] == 0 else (pos0[b] + n_tokens[b]) // C - pos0[b] // C
-        cks.append(slots[i:i + m].cpu().numpy())
-        i += m
-    return o.cpu().numpy(), state.cpu().numpy(), cks
 
 
 def _check_oracle(inp, pos0, n_tokens, S0, C, got):

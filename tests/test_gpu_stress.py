@@ -18,13 +18,14 @@ import pytest
 import oracle
 import paper_2609_15030_gb300 as hs
 from hs_inputs import gen_stress_case
-from tests.gpu_helpers import TOL, device, maxnorm_err, run_prefill
+from tests.gpu_helpers import TOL, device, maxnorm_err, run_prefill, run_scan_prefill
 
 pytestmark = pytest.mark.gpu
 
 KNOWN = [90147, 100669, 102867]
 BLOCK = 25
 BLOCKS = 12                 # 300 seeds from 200000
+SCAN_BLOCKS = 4             # 100 seeds from 210000 through the segment-parallel prefill
 
 
 def _kernels(case):
@@ -72,3 +73,36 @@ def test_seeded_stress_calls(block):
         if not e <= TOL:
             bad.append((seed, round(e, 6)))
     assert not bad, f"calls above {TOL}: {bad}"
+
+
+def _scan_error(seed, dev):
+    """Largest error of the segment-parallel prefill on stress call `seed`."""
+    c = gen_stress_case(seed)
+    x = c.inputs
+    ro, rS, rck = oracle.gla(x.q, x.k, x.v, x.a, c.pos0, c.n_tokens, S0=c.S0,
+                             C_=c.ckpt_interval, threads=16)
+    o, S, cks = run_scan_prefill(x, c.pos0, c.n_tokens, c.S0, c.ckpt_interval, dev)
+    errs = [maxnorm_err(S, rS, axes=(2, 3))]
+    for b, n in enumerate(c.n_tokens):
+        if n:
+            errs.append(maxnorm_err(o[b, :n], ro[b, :n], axes=(0, 2)))
+        assert cks[b].shape == rck[b].shape
+        if cks[b].shape[0]:
+            errs.append(maxnorm_err(cks[b], rck[b], axes=(2, 3)))
+    e = max(errs)
+    assert np.isfinite(e), seed
+    return e
+
+
+@pytest.mark.parametrize("block", range(SCAN_BLOCKS))
+def test_seeded_stress_calls_segment_parallel(block):
+    """The same kind of calls through hs_linattn_prefill_scan: its segment-state pass (tf32
+    products), the fp32 scan and the guarded output pass stay within the bar too."""
+    dev = device()
+    bad = []
+    for seed in range(210000 + BLOCK * block, 210000 + BLOCK * (block + 1)):
+        e = _scan_error(seed, dev)
+        if not e <= TOL:
+            bad.append((seed, round(e, 6)))
+    assert not bad, f"calls above {TOL}: {bad}"
+
