@@ -53,5 +53,22 @@ int main(void)
     check(hs_test_prefill_stalled(&shp, NULL, NULL, NULL, NULL, NULL, NULL, pos0, n, 0, NULL,
                                   NULL, 0) == HS_ERR_UNSUPPORTED,
           "stall hook needs the tensor-core kernel");
+
+    /* the segment-parallel prefill: its workspace, and the allocation-free variant's limit */
+    hs_linattn_shape one = {1, 16, 128, 128, 1024, HS_LINATTN_AUTO, 0};
+    const int64_t at[] = {4096};
+    const int32_t len[] = {512};
+    int64_t ws = -1;
+    check(hs_linattn_scan_workspace_bytes(&one, at, len, &ws) == HS_OK &&
+              ws == (int64_t)HS_NOALLOC_SCRATCH_BYTES,
+          "scan workspace of a 512-token tail of 16 heads = the fixed workspace");
+    check(hs_linattn_prefill_scan(&one, NULL, NULL, NULL, NULL, NULL, NULL, at, len, 512, NULL,
+                                  NULL, 0, NULL, 0) == HS_ERR_INVALID_ARG,
+          "scan prefill without a workspace");
+    const int32_t longer[] = {513};
+    check(hs_linattn_prefill_scan_noalloc(&one, NULL, NULL, NULL, NULL, NULL, NULL, at, longer, 512,
+                                          NULL, NULL, 0) == HS_ERR_TOO_LARGE &&
+              strncmp(hs_status_string(HS_ERR_TOO_LARGE), "HS_ERR_TOO_LARGE", 16) == 0,
+          "allocation-free prefill refuses a call beyond its workspace");
     return fails == 0 ? 0 : 1;
 }

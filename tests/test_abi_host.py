@@ -362,4 +362,4 @@ def test_c_client_compiles_links_and_runs(tmp_path):
                     "-o", str(exe), "-L", libdir, "-l:libhs.so", f"-Wl,-rpath,{libdir}"], check=True)
     r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
     assert r.returncode == 0, r.stdout + r.stderr
-    assert "FAIL" not in r.stdout and r.stdout.count("ok ") >= 9
+    assert "FAIL" not in r.stdout and r.stdout.count("ok ") >= 12
