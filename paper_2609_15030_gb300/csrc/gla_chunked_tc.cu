@@ -485,6 +485,13 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
     // so the next segment's state is loaded while the previous segment's products run.
     int loaded = 0;   // index of the segment whose start state is in TMEM (state warps)
     auto seg_idx = [&](int64_t at) -> int { return (int)(at / CH - pos0 / CH); };
+    // (issuing thread) the start state of the segment at `at` into L2, one bulk request
+    auto prefetch_state = [&](int64_t at) {
+        const float *src = st_g + (int64_t)seg_idx(at) * p.n_heads * D * D;
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src),
+                     "r"((uint32_t)(D * D * 4))
+                     : "memory");
+    };
     auto state_run_restart = [&](int64_t rpos, int64_t rtok) {
         int par = 0;
         bool pend = false;
@@ -518,6 +525,8 @@ gla_chunked_tc_kernel(const __grid_constant__ GlaParams p, const __grid_constant
                     return;
                 break;
             }
+            if (tid == kIssuer && is_long(rpos + L))
+                prefetch_state(rpos + L);   // read by the load at the end of this segment
             if (pend && !wait_group(2, kIssuer, bar_o, ph_o))
                 return;
             // the products of the previous segment are complete: its operand set is free
