@@ -382,8 +382,12 @@ hs_status hs_linattn_prefill_packed(const hs_linattn_shape *shp, const uint16_t 
  * kernel computes every (segment, head)'s dS and G at once (tf32 tensor-core
  * products), an elementwise scan chains S_{n+1} = G_n S_n + dS_n per (problem, head)
  * and writes the checkpoints and the final state, and the tensor-core prefill kernel
- * runs every segment again from its start state S_n for the outputs.  A call with
- * one problem of 16 heads then occupies (segments x 16) CTAs instead of 16.
+ * runs every segment again from its start state S_n for the outputs (consecutive
+ * segments grouped so that the launch fills the SMs; each segment still starts from its
+ * own S_n, so the grouping changes no result).  A call with one problem of 16 heads
+ * then spreads (segments x 16) units of work over the GPU instead of 16 chains; for
+ * calls whose (problem, head) pairs already fill the SMs it is slower than
+ * hs_linattn_prefill_from_state, which reads and writes fewer bytes.
  *
  * Results: the outputs, final states and checkpoints of the same recurrence, within
  * the same accuracy as hs_linattn_prefill_from_state (the two are not bit-identical:
