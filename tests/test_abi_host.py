@@ -299,6 +299,11 @@ def test_scan_prefill_host_validation():
             call(**kw)
         assert e.value.status == code, kw
     call(n_tokens=[0, 0], q=None, workspace=None, workspace_bytes=0)   # nothing to compute: OK
+    # (segment, head) units are 32-bit: 40,000 segments x 65,536 heads is refused
+    big = hs.make_shape(1, 65536, 128, 128, 64 * 40000)
+    with pytest.raises(hs.HsError) as e:
+        hs.hs_linattn_scan_workspace_bytes(big, [0], [64 * 40000])
+    assert e.value.status == hs.HS_ERR_UNSUPPORTED
 
 
 def test_noalloc_scan_rejects_on_the_host():
